@@ -118,6 +118,7 @@ void rsref_accept(const float *logits, long V, const int *node_off, int B,
         for (int i = 1; i < N && !bad; ++i) {
             int p = par[i];
             if (p < 0 || p >= i) { bad = 1; break; }
+            if (tok[i] < 0 || (long)tok[i] >= V) { bad = 1; break; } /* not a vocabulary id */
             if (src[i] == 1) {
                 if (src[p] > 1 || chn[i] != -1) bad = 1;
             } else if (src[i] == 2) {

@@ -1,0 +1,316 @@
+// attn.cu -- rs_tree_verify_attn: attention of the verify pass over the
+// packed draft tree (Algorithm 1 l.13 / l.25; "parallel verification" of
+// Section 3.3).  Node i of request b attends to the b's committed prefix and
+// to the tree slots of its ancestors and itself.
+//
+// Work decomposition (identical for every compute core):
+//   segment = (request b, KV head, row tile of 128 (node, q-head-in-group)
+//             rows); unit = one 128-key KV tile of a segment.
+//   The units of all segments are laid end to end and cut into gridDim.x
+//   equal ranges, one per CTA, so every SM streams the same number of KV
+//   tiles whatever the mix of context lengths (a stream-K split).  A segment
+//   that lies inside one CTA's range is finished by that CTA; a segment cut
+//   by range boundaries leaves one partial (unnormalised O, running max,
+//   running sum) per piece, in one of two slots per CTA, and the combine
+//   kernel merges them.  Nothing spins or waits across CTAs.
+//   attn_prep validates each tree and builds a 256-bit ancestor set per
+//   node; the tree part of the mask is a bit test on it.
+#include <math.h>
+
+#include "attn_core.cuh"
+#include "common.cuh"
+
+namespace rs {
+namespace {
+
+struct ReqInfo {
+    int units;  // Hkv * mt * nt, 0 for a rejected request
+    int mt;     // row tiles
+    int nt;     // KV tiles
+    int ok;
+};
+
+__global__ void __launch_bounds__(256)
+attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_len,
+          const int32_t *__restrict__ parents, int Hq, int Hkv, int D, ReqInfo *__restrict__ info,
+          uint32_t *__restrict__ anc, float *__restrict__ out, float *__restrict__ lse,
+          int32_t *__restrict__ status) {
+    const int b = blockIdx.x, tid = threadIdx.x;
+    const int n0 = node_off[b];
+    const int N = node_off[b + 1] - n0;
+    const int S = ctx_len[b];
+    const int G = Hq / Hkv;
+    __shared__ int s_par[RS_MAX_NODES];
+    __shared__ int s_bad;
+
+    int st = 0;
+    if (N < 0 || S < 0) st = RS_ST_BAD_TREE;
+    else if (N > RS_MAX_NODES) st = RS_ST_TOO_LARGE;
+    if (tid == 0) s_bad = 0;
+    __syncthreads();
+    if (st == 0) {
+        for (int i = tid; i < N; i += blockDim.x) {
+            int pa = parents[n0 + i];
+            s_par[i] = pa;
+            if (i == 0 ? pa != -1 : (pa < 0 || pa >= i)) atomicOr(&s_bad, 1);
+        }
+        __syncthreads();
+        if (s_bad) st = RS_ST_BAD_TREE;
+    }
+    if (st == 0) {
+        for (int i = tid; i < N; i += blockDim.x) {
+            uint32_t bits[kAncWords];
+#pragma unroll
+            for (int w = 0; w < kAncWords; ++w) bits[w] = 0;
+            for (int a = i; a >= 0; a = s_par[a]) bits[a >> 5] |= 1u << (a & 31);
+#pragma unroll
+            for (int w = 0; w < kAncWords; ++w) anc[(long long)(n0 + i) * kAncWords + w] = bits[w];
+        }
+        if (tid == 0) {
+            int mt = (N * G + kBM - 1) / kBM;
+            int nt = (S + N + kBN - 1) / kBN;
+            info[b] = ReqInfo{Hkv * mt * nt, mt, nt, 1};
+        }
+    } else {
+        if (tid == 0) info[b] = ReqInfo{0, 0, 0, 0};
+        if (N > 0) {
+            const long long n = (long long)N * Hq;
+            for (long long x = tid; x < n * D; x += blockDim.x) out[(long long)n0 * Hq * D + x] = 0.f;
+            for (long long x = tid; x < n; x += blockDim.x) lse[(long long)n0 * Hq + x] = 0.f;
+        }
+    }
+    if (tid == 0) status[b] = st;
+}
+
+// Exclusive prefix of per-request units into s_pref[0..B] (s_pref[B] = W).
+__device__ void unit_prefix(const ReqInfo *__restrict__ info, int B, int *s_pref) {
+    __shared__ int s_carry;
+    if (threadIdx.x == 0) s_carry = 0;
+    __syncthreads();
+    for (int base = 0; base < B; base += blockDim.x) {
+        int i = base + threadIdx.x;
+        int v = i < B ? info[i].units : 0;
+        // inclusive warp scan, then across warps (blockDim.x <= 1024)
+        __shared__ int s_w[32];
+        int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+        int x = v;
+        for (int o = 1; o < 32; o <<= 1) {
+            int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        if (lane == 31) s_w[warp] = x;
+        __syncthreads();
+        if (warp == 0) {
+            int nw = (blockDim.x + 31) >> 5;
+            int w = lane < nw ? s_w[lane] : 0;
+            int z = w;
+            for (int o = 1; o < 32; o <<= 1) {
+                int y = __shfl_up_sync(0xffffffffu, z, o);
+                if (lane >= o) z += y;
+            }
+            s_w[lane] = z - w;
+        }
+        __syncthreads();
+        int incl = s_carry + s_w[warp] + x;
+        if (i < B) s_pref[i + 1] = incl;
+        __syncthreads();
+        if (threadIdx.x == blockDim.x - 1) s_carry = incl;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) s_pref[0] = 0;
+    __syncthreads();
+}
+
+// last b with s_pref[b] <= u (requests with no units are skipped)
+__device__ __forceinline__ int find_req(const int *s_pref, int B, long long u) {
+    int lo = 0, hi = B - 1;
+    while (lo < hi) {
+        int mid = (lo + hi + 1) >> 1;
+        if (s_pref[mid] <= u) lo = mid;
+        else hi = mid - 1;
+    }
+    while (lo + 1 <= B - 1 && s_pref[lo + 1] <= u) ++lo;
+    return lo;
+}
+
+__device__ __forceinline__ long long range_lo(long long c, long long W, long long G) { return c * W / G; }
+__device__ __forceinline__ long long owner_of(long long u, long long W, long long G) {
+    return ((u + 1) * G - 1) / W;
+}
+
+__global__ void __launch_bounds__(kAttnThreads)
+attn_main(AttnArgs a, const ReqInfo *__restrict__ info) {
+    extern __shared__ __align__(1024) unsigned char smem[];
+    int *s_pref = reinterpret_cast<int *>(smem + kAttnSmemTiles);
+    unit_prefix(info, a.B, s_pref);
+    const long long W = s_pref[a.B];
+    const long long Gc = gridDim.x, c = blockIdx.x;
+    const long long u0 = range_lo(c, W, Gc), u1 = range_lo(c + 1, W, Gc);
+    long long u = u0;
+    while (u < u1) {
+        const int b = find_req(s_pref, a.B, u);
+        const ReqInfo ri = info[b];
+        const long long local = u - s_pref[b];
+        const int seg = (int)(local / ri.nt);
+        const int j0 = (int)(local - (long long)seg * ri.nt);
+        const long long seg_start = s_pref[b] + (long long)seg * ri.nt;
+        const long long seg_end = seg_start + ri.nt;
+        const long long pend = seg_end < u1 ? seg_end : u1;
+        Piece pc;
+        pc.b = b;
+        pc.kvh = seg / ri.mt;
+        pc.mtile = seg - pc.kvh * ri.mt;
+        pc.j0 = j0;
+        pc.j1 = j0 + (int)(pend - u);
+        pc.final = (seg_start >= u0 && seg_end <= u1);
+        pc.slot = (int)(2 * c + (seg_start > u0 ? 1 : 0));
+        attn_piece(a, pc, smem);
+        u = pend;
+    }
+}
+
+__global__ void __launch_bounds__(256)
+attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
+    extern __shared__ int s_pref[];
+    unit_prefix(info, a.B, s_pref);
+    const long long W = s_pref[a.B];
+    const long long Gc = gridDim.x, c = blockIdx.x;
+    const long long u0 = range_lo(c, W, Gc), u1 = range_lo(c + 1, W, Gc);
+    if (u0 >= u1) return;
+    const int b = find_req(s_pref, a.B, u1 - 1);
+    const ReqInfo ri = info[b];
+    const long long local = u1 - 1 - s_pref[b];
+    const int seg = (int)(local / ri.nt);
+    const long long seg_start = s_pref[b] + (long long)seg * ri.nt;
+    const long long seg_end = seg_start + ri.nt;
+    if (!(seg_start >= u0 && seg_end > u1)) return;  // not the first owner of a split segment
+    const long long c1 = owner_of(seg_end - 1, W, Gc);
+
+    const int G = a.Hq / a.Hkv;
+    const int n0 = a.node_off[b];
+    const int N = a.node_off[b + 1] - n0;
+    const int kvh = seg / ri.mt, mtile = seg - kvh * ri.mt;
+    const int rows = min(kBM, N * G - mtile * kBM);
+    const int D = a.D;
+    for (int x = threadIdx.x; x < rows * D; x += blockDim.x) {
+        const int r = x / D, d = x - r * D;
+        float M = -INFINITY;
+        for (long long cc = c; cc <= c1; ++cc) {
+            const long long lo = range_lo(cc, W, Gc);
+            if (lo == range_lo(cc + 1, W, Gc)) continue;
+            const int slot = (int)(2 * cc + (seg_start > lo ? 1 : 0));
+            M = fmaxf(M, a.part_m[(long long)slot * kBM + r]);
+        }
+        float L = 0.f, O = 0.f;
+        for (long long cc = c; cc <= c1; ++cc) {
+            const long long lo = range_lo(cc, W, Gc);
+            if (lo == range_lo(cc + 1, W, Gc)) continue;
+            const int slot = (int)(2 * cc + (seg_start > lo ? 1 : 0));
+            const float m = a.part_m[(long long)slot * kBM + r];
+            if (m == -INFINITY) continue;
+            const float w = __expf(m - M);
+            L += w * a.part_l[(long long)slot * kBM + r];
+            O += w * a.part_o[((long long)slot * kBM + r) * D + d];
+        }
+        const int rr = mtile * kBM + r;
+        const int i = rr / G, h = kvh * G + (rr - (rr / G) * G);
+        const long long orow = (long long)(n0 + i) * a.Hq + h;
+        a.out[orow * D + d] = O / L;
+        if (d == 0) a.lse[orow] = M + __logf(L);
+    }
+}
+
+int g_attr_done[64] = {0};
+
+}  // namespace
+}  // namespace rs
+
+using namespace rs;
+
+static int attn_grid() { return num_sms() * kAttnCtasPerSm; }
+
+extern "C" size_t rs_tree_verify_attn_workspace_size(int B, int R, int Hq, int Hkv, int D) {
+    if (B < 0 || R < 0 || Hq < 1 || Hkv < 1 || (D != 64 && D != 128)) return 0;
+    const size_t Gc = (size_t)attn_grid();
+    Carve cv(nullptr);
+    cv.take<ReqInfo>((size_t)B);
+    cv.take<uint32_t>((size_t)R * kAncWords);
+    cv.take<float>(2 * Gc * kBM * (size_t)D);
+    cv.take<float>(2 * Gc * kBM);
+    cv.take<float>(2 * Gc * kBM);
+    return cv.used();
+}
+
+extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, const uint16_t *v, int64_t kv_rows,
+                                         const int64_t *kv_off, const int32_t *ctx_len, const int32_t *node_off,
+                                         const int32_t *parents, int B, int R, int Hq, int Hkv, int D, float scale,
+                                         float *out, float *lse, int32_t *status, void *workspace,
+                                         size_t workspace_bytes, void *stream) {
+    clear_error();
+    RS_CHECK_ARG(B >= 0 && R >= 0 && kv_rows >= 0, "rs_tree_verify_attn: negative size");
+    if (D != 64 && D != 128) {
+        set_error("rs_tree_verify_attn: head dim %d unsupported (64 or 128)", D);
+        return RS_ERR_UNSUPPORTED;
+    }
+    if (Hkv < 1 || Hq < 1 || Hq % Hkv != 0) {
+        set_error("rs_tree_verify_attn: Hq=%d must be a positive multiple of Hkv=%d", Hq, Hkv);
+        return RS_ERR_UNSUPPORTED;
+    }
+    RS_CHECK_ARG(B <= 16384, "rs_tree_verify_attn: B=%d above 16384", B);
+    RS_CHECK_ARG(isfinite(scale), "rs_tree_verify_attn: scale must be finite");
+    RS_CHECK_ARG(B == 0 || (kv_off && ctx_len && node_off && status), "rs_tree_verify_attn: null request pointer");
+    RS_CHECK_ARG(R == 0 || (q && parents && out && lse), "rs_tree_verify_attn: null row pointer");
+    RS_CHECK_ARG(kv_rows == 0 || (k && v), "rs_tree_verify_attn: null KV pointer");
+    RS_CHECK_ARG((((uintptr_t)k | (uintptr_t)v | (uintptr_t)q) & 15) == 0,
+                 "rs_tree_verify_attn: q, k and v must be 16-byte aligned");
+    if (B == 0) return RS_OK;
+    const size_t need = rs_tree_verify_attn_workspace_size(B, R, Hq, Hkv, D);
+    if (workspace_bytes < need || !workspace) {
+        set_error("rs_tree_verify_attn: workspace %zu bytes < %zu required", workspace_bytes, need);
+        return RS_ERR_CAPACITY;
+    }
+    const int Gc = attn_grid();
+    Carve cv(workspace);
+    ReqInfo *info = cv.take<ReqInfo>((size_t)B);
+    uint32_t *anc = cv.take<uint32_t>((size_t)R * kAncWords);
+    AttnArgs a;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.kv_off = kv_off;
+    a.ctx_len = ctx_len;
+    a.node_off = node_off;
+    a.anc = anc;
+    a.part_o = cv.take<float>(2 * (size_t)Gc * kBM * D);
+    a.part_m = cv.take<float>(2 * (size_t)Gc * kBM);
+    a.part_l = cv.take<float>(2 * (size_t)Gc * kBM);
+    a.B = B;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.D = D;
+    a.scale = scale;
+    a.out = out;
+    a.lse = lse;
+    cudaStream_t st = (cudaStream_t)stream;
+
+    attn_prep<<<B, 256, 0, st>>>(node_off, ctx_len, parents, Hq, Hkv, D, info, anc, out, lse, status);
+    RS_CHECK_LAUNCH("rs_tree_verify_attn/prep");
+
+    const size_t smem_main = kAttnSmemTiles + (size_t)(B + 1) * sizeof(int);
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !g_attr_done[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(attn_main, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kAttnSmemTiles + (16384 + 1) * (int)sizeof(int));
+        if (e != cudaSuccess) {
+            set_error("rs_tree_verify_attn: cudaFuncSetAttribute: %s", cudaGetErrorString(e));
+            return RS_ERR_CUDA;
+        }
+        g_attr_done[dev] = 1;
+    }
+    attn_main<<<Gc, kAttnThreads, smem_main, st>>>(a, info);
+    RS_CHECK_LAUNCH("rs_tree_verify_attn/main");
+    attn_combine<<<Gc, 256, (size_t)(B + 1) * sizeof(int), st>>>(a, info);
+    RS_CHECK_LAUNCH("rs_tree_verify_attn/combine");
+    return RS_OK;
+}

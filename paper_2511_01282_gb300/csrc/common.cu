@@ -1,0 +1,48 @@
+// common.cu -- error reporting, version and launch accounting of the library.
+#include <atomic>
+#include <mutex>
+
+#include "common.cuh"
+
+namespace rs {
+
+static thread_local char g_err[1024] = "";
+static std::atomic<uint64_t> g_launches{0};
+
+void set_error(const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof g_err, fmt, ap);
+    va_end(ap);
+}
+
+void clear_error() { g_err[0] = 0; }
+
+void count_launch(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+int num_sms() {
+    static std::mutex mu;
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+    std::lock_guard<std::mutex> lk(mu);
+    if (!cache[dev]) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+            n = 148;
+        cache[dev] = n;
+    }
+    return cache[dev];
+}
+
+}  // namespace rs
+
+extern "C" {
+
+const char *rs_last_error(void) { return rs::g_err; }
+
+const char *rs_version(void) { return "respec-gb300 0.1 (sm_103a)"; }
+
+uint64_t rs_launch_count(void) { return rs::g_launches.load(); }
+
+}  // extern "C"

@@ -1,0 +1,94 @@
+// common.cuh -- shared helpers of the sm_103a ReSpec library (host checks,
+// error reporting, launch accounting, warp/block reductions).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <stdio.h>
+
+#include <cstdarg>
+
+#include "respec.h"
+
+namespace rs {
+
+// ---------------------------------------------------------------- host side
+void set_error(const char *fmt, ...);
+void clear_error();
+void count_launch(int n = 1);
+
+#define RS_CHECK_ARG(cond, ...)                            \
+    do {                                                   \
+        if (!(cond)) {                                     \
+            ::rs::set_error(__VA_ARGS__);                  \
+            return RS_ERR_INVALID_ARG;                     \
+        }                                                  \
+    } while (0)
+
+#define RS_CHECK_LAUNCH(what)                                                        \
+    do {                                                                             \
+        cudaError_t e_ = cudaGetLastError();                                         \
+        if (e_ != cudaSuccess) {                                                     \
+            ::rs::set_error("%s: launch failed: %s", what, cudaGetErrorString(e_));  \
+            return RS_ERR_CUDA;                                                      \
+        }                                                                            \
+        ::rs::count_launch();                                                        \
+    } while (0)
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Bump allocator over the caller's workspace (256-byte aligned slices).
+struct Carve {
+    char *base;
+    size_t off = 0;
+    explicit Carve(void *p) : base(static_cast<char *>(p)) {}
+    template <class T>
+    T *take(size_t n) {
+        off = align_up(off, 256);
+        T *p = reinterpret_cast<T *>(base ? base + off : nullptr);
+        off += n * sizeof(T);
+        return p;
+    }
+    size_t used() const { return align_up(off, 256); }
+};
+
+int num_sms();  // SM count of the current device (cached per device)
+
+// ---------------------------------------------------------------- device side
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ int warp_sum_i(int v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// (value, id) total order used for argmax / TopK: larger value first, then
+// smaller id.  Returns true when (va, ia) comes strictly before (vb, ib).
+__device__ __forceinline__ bool vi_before(float va, int ia, float vb, int ib) {
+    return va > vb || (va == vb && ia < ib);
+}
+
+// Read-only, L1-bypassing streaming loads for data read exactly once.
+__device__ __forceinline__ float4 ldg_stream4(const float4 *p) {
+    float4 r;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0,%1,%2,%3}, [%4];"
+                 : "=f"(r.x), "=f"(r.y), "=f"(r.z), "=f"(r.w)
+                 : "l"(p));
+    return r;
+}
+__device__ __forceinline__ float ldg_stream(const float *p) {
+    float r;
+    asm volatile("ld.global.nc.L1::no_allocate.f32 %0, [%1];" : "=f"(r) : "l"(p));
+    return r;
+}
+
+}  // namespace rs

@@ -1,0 +1,225 @@
+// gate.cu -- rs_entropy_gate: entropy-guided adaptive trigger
+// (Section 3.2.1, Eq. 1-3 and step 4; Algorithm 1 step 1).
+//
+// Kernel 1 (entropy_partial): one CTA per (row, 8192-logit chunk).  Each
+// thread streams 32 logits with 128-bit loads and forms, relative to its own
+// maximum m, s = sum e^(z-m) and w = sum e^(z-m) (z-m); the CTA merges the
+// triples with warp shuffles and writes one triple per chunk.  Row entropy
+// is then H = ln s - w / s for the merged triple (the log-sum-exp form of
+// -sum p ln p).
+// Kernel 2 (gate_finalize): one CTA per request merges its rows' chunk
+// triples, writes the row entropies, pushes the committed rows into the
+// history and evaluates H_k, C_k, k* and the trigger in fp64.
+#include <math.h>
+
+#include "common.cuh"
+
+namespace rs {
+namespace {
+
+constexpr int kGateThreads = 256;
+constexpr int kGateVpt = 32;                          // logits per thread
+constexpr int kGateChunk = kGateThreads * kGateVpt;   // logits per CTA
+
+struct Ent3 {
+    float m, s, w;
+};
+
+__device__ __forceinline__ Ent3 ent_merge(Ent3 a, Ent3 b) {
+    if (a.s == 0.f) return b;
+    if (b.s == 0.f) return a;
+    float M = fmaxf(a.m, b.m);
+    float ca = __expf(a.m - M), cb = __expf(b.m - M);
+    Ent3 r;
+    r.m = M;
+    r.s = a.s * ca + b.s * cb;
+    r.w = ca * (a.w + a.s * (a.m - M)) + cb * (b.w + b.s * (b.m - M));
+    return r;
+}
+
+__device__ __forceinline__ Ent3 ent_shfl(Ent3 a, int o) {
+    Ent3 b;
+    b.m = __shfl_xor_sync(0xffffffffu, a.m, o);
+    b.s = __shfl_xor_sync(0xffffffffu, a.s, o);
+    b.w = __shfl_xor_sync(0xffffffffu, a.w, o);
+    return b;
+}
+
+// One thread's triple over its kGateVpt values (-inf padded).
+__device__ __forceinline__ Ent3 ent_local(const float (&v)[kGateVpt]) {
+    float mx = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < kGateVpt; ++i) mx = fmaxf(mx, v[i]);
+    Ent3 r{mx, 0.f, 0.f};
+    if (mx == -INFINITY) return r;
+#pragma unroll
+    for (int i = 0; i < kGateVpt; ++i) {
+        float d = fmaxf(v[i] - mx, -1e30f);  // -inf -> -1e30: e = 0, e*d = 0
+        float e = __expf(d);
+        r.s += e;
+        r.w = fmaf(e, d, r.w);
+    }
+    return r;
+}
+
+template <bool kVec>
+__global__ void __launch_bounds__(kGateThreads)
+entropy_partial(const float *__restrict__ logits, int V, int nchunks, Ent3 *__restrict__ part) {
+    const long long blk = blockIdx.x;
+    const long long r = blk / nchunks;
+    const int chunk = (int)(blk - r * nchunks);
+    const float *row = logits + r * (long long)V;
+    const int c0 = chunk * kGateChunk;
+    const int tid = threadIdx.x;
+
+    float v[kGateVpt];
+    if (kVec) {
+        // 8 x float4 per thread, each iteration a contiguous 4 KB sweep
+#pragma unroll
+        for (int j = 0; j < kGateVpt / 4; ++j) {
+            int idx = c0 + (j * kGateThreads + tid) * 4;
+            float4 x;
+            if (idx + 3 < V) {
+                x = ldg_stream4(reinterpret_cast<const float4 *>(row + idx));
+            } else {
+                x.x = idx + 0 < V ? row[idx + 0] : -INFINITY;
+                x.y = idx + 1 < V ? row[idx + 1] : -INFINITY;
+                x.z = idx + 2 < V ? row[idx + 2] : -INFINITY;
+                x.w = -INFINITY;
+            }
+            v[4 * j + 0] = x.x;
+            v[4 * j + 1] = x.y;
+            v[4 * j + 2] = x.z;
+            v[4 * j + 3] = x.w;
+        }
+    } else {
+#pragma unroll
+        for (int j = 0; j < kGateVpt; ++j) {
+            int idx = c0 + j * kGateThreads + tid;
+            v[j] = idx < V ? ldg_stream(row + idx) : -INFINITY;
+        }
+    }
+
+    Ent3 t = ent_local(v);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t = ent_merge(t, ent_shfl(t, o));
+    __shared__ Ent3 sw[kGateThreads / 32];
+    if ((tid & 31) == 0) sw[tid >> 5] = t;
+    __syncthreads();
+    if (tid < 32) {
+        t = tid < kGateThreads / 32 ? sw[tid] : Ent3{-INFINITY, 0.f, 0.f};
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) t = ent_merge(t, ent_shfl(t, o));
+        if (tid == 0) part[blk] = t;
+    }
+}
+
+__global__ void __launch_bounds__(256)
+gate_finalize(const Ent3 *__restrict__ part, int nchunks, const int32_t *__restrict__ row_off,
+              const uint8_t *__restrict__ row_commit, rs_params p, float *__restrict__ hist,
+              int32_t *__restrict__ hist_n, float *__restrict__ entropy, int32_t *__restrict__ k_star,
+              float *__restrict__ h_best, uint8_t *__restrict__ entropy_ok) {
+    const int b = blockIdx.x;
+    const int r0 = row_off[b], r1 = row_off[b + 1];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+
+    // row entropies: one warp per row, lanes over chunks
+    for (int r = r0 + warp; r < r1; r += blockDim.x >> 5) {
+        Ent3 t{-INFINITY, 0.f, 0.f};
+        for (int c = lane; c < nchunks; c += 32) t = ent_merge(t, part[(long long)r * nchunks + c]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) t = ent_merge(t, ent_shfl(t, o));
+        if (lane == 0) entropy[r] = t.s > 0.f ? (__logf(t.s) - t.w / t.s) : 0.f;
+    }
+    __syncthreads();  // this block's entropy[] writes are visible below
+
+    if (threadIdx.x != 0) return;
+    const int l = p.l;
+    float h[RS_MAX_L];
+    int n = hist_n[b];
+    n = n < 0 ? 0 : (n > l ? l : n);
+    for (int i = 0; i < l; ++i) h[i] = hist[(long long)b * l + i];
+    for (int r = r0; r < r1; ++r) {
+        if (!row_commit[r]) continue;
+        float e = entropy[r];
+        if (n == l) {
+            for (int i = 1; i < l; ++i) h[i - 1] = h[i];
+            h[l - 1] = e;
+        } else {
+            h[n++] = e;
+        }
+    }
+    for (int i = 0; i < l; ++i) hist[(long long)b * l + i] = h[i];
+    hist_n[b] = n;
+
+    // Algorithm 1 step 1 in fp64: k upward, strict '<'
+    double c_min = INFINITY, best = INFINITY;
+    int kbest = 0;
+    for (int k = 1; k <= n; ++k) {
+        double s = 0.0;
+        for (int i = n - k; i < n; ++i) s = __dadd_rn(s, (double)h[i]);
+        double hk = __ddiv_rn(s, (double)k);
+        double ck = __dadd_rn(hk, __ddiv_rn((double)p.lambda_e, (double)k));
+        if (ck < c_min) {
+            c_min = ck;
+            best = hk;
+            kbest = k;
+        }
+    }
+    k_star[b] = kbest;
+    h_best[b] = (float)best;
+    entropy_ok[b] = (uint8_t)(kbest > 0 && best <= (double)p.theta_entropy);
+}
+
+}  // namespace
+}  // namespace rs
+
+using namespace rs;
+
+extern "C" size_t rs_entropy_gate_workspace_size(int R, int V) {
+    if (R < 0 || V < 1) return 0;
+    int nchunks = (V + kGateChunk - 1) / kGateChunk;
+    Carve cv(nullptr);
+    cv.take<Ent3>((size_t)R * nchunks);
+    return cv.used();
+}
+
+extern "C" rs_status rs_entropy_gate(const float *logits, int R, int V, const int32_t *row_off,
+                                     const uint8_t *row_commit, int B, rs_params p, float *hist,
+                                     int32_t *hist_n, float *entropy, int32_t *k_star, float *h_best,
+                                     uint8_t *entropy_ok, void *workspace, size_t workspace_bytes,
+                                     void *stream) {
+    clear_error();
+    RS_CHECK_ARG(R >= 0 && B >= 0, "rs_entropy_gate: negative size (R=%d, B=%d)", R, B);
+    RS_CHECK_ARG(V >= 1, "rs_entropy_gate: V must be >= 1 (got %d)", V);
+    RS_CHECK_ARG(p.l >= 1 && p.l <= RS_MAX_L, "rs_entropy_gate: l=%d outside [1, %d]", p.l, RS_MAX_L);
+    RS_CHECK_ARG(R == 0 || (logits && entropy && row_commit), "rs_entropy_gate: null row pointer");
+    RS_CHECK_ARG(B == 0 || (row_off && hist && hist_n && k_star && h_best && entropy_ok),
+                 "rs_entropy_gate: null request pointer");
+    const int nchunks = (V + kGateChunk - 1) / kGateChunk;
+    const size_t need = rs_entropy_gate_workspace_size(R, V);
+    if (workspace_bytes < need || (need && !workspace)) {
+        set_error("rs_entropy_gate: workspace %zu bytes < %zu required", workspace_bytes, need);
+        return RS_ERR_CAPACITY;
+    }
+    cudaStream_t st = (cudaStream_t)stream;
+    Carve cv(workspace);
+    Ent3 *part = cv.take<Ent3>((size_t)R * nchunks);
+
+    if (R > 0) {
+        long long blocks = (long long)R * nchunks;
+        RS_CHECK_ARG(blocks < (1ll << 31), "rs_entropy_gate: R*chunks too large");
+        bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
+        if (vec)
+            entropy_partial<true><<<(unsigned)blocks, kGateThreads, 0, st>>>(logits, V, nchunks, part);
+        else
+            entropy_partial<false><<<(unsigned)blocks, kGateThreads, 0, st>>>(logits, V, nchunks, part);
+        RS_CHECK_LAUNCH("rs_entropy_gate/entropy_partial");
+    }
+    if (B > 0) {
+        gate_finalize<<<B, 256, 0, st>>>(part, nchunks, row_off, row_commit, p, hist, hist_n, entropy,
+                                         k_star, h_best, entropy_ok);
+        RS_CHECK_LAUNCH("rs_entropy_gate/gate_finalize");
+    }
+    return RS_OK;
+}

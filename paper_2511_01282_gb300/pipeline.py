@@ -1,0 +1,143 @@
+"""One verify-and-draft step on the GPU, as the four C-ABI calls.
+
+``VerifyStep`` owns the device buffers of one batch (inputs, outputs and the
+per-call workspaces, all plain torch allocations) and enqueues, on one
+stream, the calls of one step of Algorithm 1 in their data-flow order:
+
+    rs_entropy_gate -> rs_match_scan (keyed by k*, gated by the trigger)
+                    -> rs_tree_verify_attn -> rs_accept
+
+It computes nothing itself.  Inputs come as host numpy arrays (bf16 as
+uint16 bit patterns) with the layouts ``include/respec.h`` documents.
+"""
+import numpy as np
+import torch
+
+from . import respec as rs
+
+
+def _dev(a, device):
+    return torch.from_numpy(np.ascontiguousarray(a)).to(device)
+
+
+class VerifyStep:
+    INPUTS = ("logits", "row_off", "row_commit", "hist", "hist_n", "tokens", "tok_off", "scores",
+              "q", "k", "v", "kv_off", "ctx_len", "node_off", "parents", "tree_tokens", "source",
+              "chain", "sel_pos")
+
+    def __init__(self, arrays, p, Hq, Hkv, D, pos_cap=1024, acc_cap=64, device="cuda",
+                 scale=None, pinned_host=False):
+        self.p = p
+        self.Hq, self.Hkv, self.D = Hq, Hkv, D
+        self.scale = float(D ** -0.5 if scale is None else scale)
+        self.pos_cap, self.acc_cap = pos_cap, acc_cap
+        self.device = torch.device(device)
+        host = dict(arrays)
+        host["row_off"] = np.asarray(host["node_off"], np.int32)
+        self.host = {k: np.ascontiguousarray(host[k]) for k in self.INPUTS}
+        self.B = int(self.host["node_off"].size - 1)
+        self.R = int(self.host["node_off"][-1])
+        self.V = int(self.host["logits"].shape[1])
+        self.kv_rows = int(self.host["k"].shape[0])
+        # device inputs
+        self.d = {k: _dev(v, self.device) for k, v in self.host.items()}
+        self.pinned = None
+        if pinned_host:
+            self.pinned = {k: torch.from_numpy(v).pin_memory() for k, v in self.host.items()}
+        B, R, V = self.B, self.R, self.V
+        dev = self.device
+        z = lambda n, dt: torch.zeros(n, dtype=dt, device=dev)  # noqa: E731
+        tc, L = p.top_c, p.span_len
+        self.out = dict(
+            entropy=z(R, torch.float32), k_star=z(B, torch.int32), h_best=z(B, torch.float32),
+            entropy_ok=z(B, torch.uint8),
+            count=z(B, torch.int32), pos=z((B, pos_cap), torch.int32), sel_pos=z((B, tc), torch.int32),
+            sel_len=z((B, tc), torch.int32), spans=z((B, tc, L), torch.int32), n_sel=z(B, torch.int32),
+            scan_status=z(B, torch.int32),
+            attn_out=z((R, Hq, D), torch.float32), attn_lse=z((R, Hq), torch.float32),
+            attn_status=z(B, torch.int32),
+            argmax=z(R, torch.int32), topk=z((R, p.beta), torch.int32), lse=z(R, torch.float32),
+            p_tok=z(R, torch.float32), acc_len=z(B, torch.int32), acc_nodes=z((B, acc_cap), torch.int32),
+            bonus=z(B, torch.int32), winner=z(B, torch.int32), commit=z(R, torch.uint8),
+            acc_status=z(B, torch.int32))
+        self.ws = dict(
+            gate=z(max(rs.rs_entropy_gate_workspace_size(R, V), 256), torch.uint8),
+            scan=z(max(rs.rs_match_scan_workspace_size(B), 256), torch.uint8),
+            attn=z(max(rs.rs_tree_verify_attn_workspace_size(B, R, Hq, Hkv, D), 256), torch.uint8),
+            accept=z(max(rs.rs_accept_workspace_size(R, V, p.beta), 256), torch.uint8))
+
+    # ------------------------------------------------------------ the calls
+    def gate(self, stream=None):
+        d, o = self.d, self.out
+        rs.rs_entropy_gate(d["logits"], self.R, self.V, d["row_off"], d["row_commit"], self.B, self.p,
+                           d["hist"], d["hist_n"], o["entropy"], o["k_star"], o["h_best"],
+                           o["entropy_ok"], self.ws["gate"], stream)
+
+    def scan(self, k_star=None, gate_ok="gate", stream=None):
+        d, o = self.d, self.out
+        ks = o["k_star"] if k_star is None else k_star
+        ok = o["entropy_ok"] if gate_ok == "gate" else gate_ok
+        rs.rs_match_scan(d["tokens"], d["tok_off"], self.B, ks, ok, d["scores"], self.p, self.pos_cap,
+                         o["count"], o["pos"], o["sel_pos"], o["sel_len"], o["spans"], o["n_sel"],
+                         o["scan_status"], self.ws["scan"], stream)
+
+    def attn(self, stream=None):
+        d, o = self.d, self.out
+        rs.rs_tree_verify_attn(d["q"], d["k"], d["v"], self.kv_rows, d["kv_off"], d["ctx_len"],
+                               d["node_off"], d["parents"], self.B, self.R, self.Hq, self.Hkv, self.D,
+                               self.scale, o["attn_out"], o["attn_lse"], o["attn_status"],
+                               self.ws["attn"], stream)
+
+    def accept(self, sel_pos=None, stream=None):
+        d, o = self.d, self.out
+        sp = d["sel_pos"] if sel_pos is None else sel_pos
+        rs.rs_accept(d["logits"], self.R, self.V, d["node_off"], self.B, d["tree_tokens"], d["parents"],
+                     d["source"], d["chain"], sp, d["tok_off"], self.p, self.acc_cap, o["argmax"],
+                     o["topk"], o["lse"], o["p_tok"], o["acc_len"], o["acc_nodes"], o["bonus"],
+                     o["winner"], o["commit"], d["scores"], o["acc_status"], self.ws["accept"], stream)
+
+    def step(self, stream=None):
+        """One pass of the whole hot path (4 calls, 9 kernel launches)."""
+        self.gate(stream)
+        self.scan(stream=stream)
+        self.attn(stream)
+        self.accept(stream=stream)
+
+    # ------------------------------------------------------ host round trip
+    def upload(self, stream=None):
+        """Copy every input from pinned host memory (async on `stream`)."""
+        s = torch.cuda.current_stream() if stream is None else stream
+        with torch.cuda.stream(s):
+            for k, t in self.pinned.items():
+                self.d[k].copy_(t, non_blocking=True)
+        return sum(t.numel() * t.element_size() for t in self.pinned.values())
+
+    RESULT_KEYS = ("acc_len", "acc_nodes", "bonus", "winner", "commit", "k_star", "entropy_ok",
+                   "sel_pos", "n_sel")
+
+    def download_into(self, host_bufs, stream=None):
+        """Copy the step's decisions to pinned host buffers (async)."""
+        s = torch.cuda.current_stream() if stream is None else stream
+        n = 0
+        with torch.cuda.stream(s):
+            for k in self.RESULT_KEYS:
+                host_bufs[k].copy_(self.out[k], non_blocking=True)
+                n += self.out[k].numel() * self.out[k].element_size()
+        return n
+
+    def result_buffers(self):
+        return {k: torch.empty(self.out[k].shape, dtype=self.out[k].dtype).pin_memory()
+                for k in self.RESULT_KEYS}
+
+    def reset_state(self):
+        """Restore the in/out state (history, scores) to the host inputs."""
+        for k in ("hist", "hist_n", "scores"):
+            self.d[k].copy_(torch.from_numpy(self.host[k]))
+
+
+def arrays_from_workload(w):
+    """Map a synthetic workload's fields onto the step's input names."""
+    return dict(logits=w.logits, node_off=w.node_off, row_commit=w.row_commit, hist=w.hist,
+                hist_n=w.hist_n, tokens=w.tokens, tok_off=w.tok_off, scores=w.scores, q=w.q, k=w.k,
+                v=w.v, kv_off=w.kv_off, ctx_len=w.ctx_len, parents=w.parents,
+                tree_tokens=w.tree_tokens, source=w.source, chain=w.chain, sel_pos=w.sel_pos)

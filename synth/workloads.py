@@ -25,7 +25,9 @@ Recipe (per request b, generator PCG64(seed * 1000 + b)):
   per row: its logit is set to the row max + U(0.1, 1)), "close" (prob 0.2:
   row max - U(0, tau)) or left alone; optionally a tie at the row maximum is
   injected at another id;
-* Q [N, Hq, D], K and V [S + N, Hkv, D]: N(0, 1) rounded to bf16;
+* Q [N, Hq, D], K and V [S + N, Hkv, D]: N(0, 1) rounded to bf16 (K and V
+  in 2048-row chunks, each from its own PCG64 stream seeded by (seed,
+  request, tensor, chunk), generated in parallel);
 * score table parallel to the buffer: 0.5 (the paper's S0), with a share of
   positions redrawn uniform in [0, 1] so the threshold filter and the ranking
   both have work to do;
@@ -37,8 +39,10 @@ acceptance decision.
 """
 from __future__ import annotations
 
+import concurrent.futures as cf
 import dataclasses
 import math
+import os
 from functools import lru_cache
 from typing import Optional, Sequence
 
@@ -46,11 +50,18 @@ import numpy as np
 
 
 # --------------------------------------------------------------------- bf16
-def bf16_bits(x: np.ndarray) -> np.ndarray:
-    """fp32 -> bf16 bit patterns (uint16), round to nearest even."""
+def bf16_bits(x: np.ndarray, out: Optional[np.ndarray] = None) -> np.ndarray:
+    """fp32 -> bf16 bit patterns (uint16), round to nearest even (finite inputs)."""
     u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
-    r = ((u >> np.uint32(16)) & np.uint32(1)) + np.uint32(0x7FFF)
-    return ((u + r) >> np.uint32(16)).astype(np.uint16)
+    r = np.right_shift(u, 16)
+    np.bitwise_and(r, 1, out=r)
+    np.add(r, 0x7FFF, out=r)
+    np.add(r, u, out=r)
+    np.right_shift(r, 16, out=r)
+    if out is None:
+        return r.astype(np.uint16)
+    np.copyto(out, r.reshape(out.shape), casting="unsafe")
+    return out
 
 
 def bf16_to_f32(h: np.ndarray) -> np.ndarray:
@@ -169,6 +180,30 @@ class Workload:
 
     def params(self):
         return self.spec.params()
+
+
+_KV_CHUNK_ROWS = 2048
+
+
+def _fill_normal_bf16(dst: np.ndarray, key: tuple):
+    """dst[...] = N(0, 1) rounded to bf16, in row chunks generated in parallel;
+    chunk j uses PCG64(SeedSequence(key + (j,))), so the values do not depend
+    on the number of threads."""
+    rows = dst.shape[0]
+    chunks = list(range(0, rows, _KV_CHUNK_ROWS))
+
+    def work(j0):
+        n = min(_KV_CHUNK_ROWS, rows - j0)
+        g = np.random.Generator(np.random.PCG64(np.random.SeedSequence(list(key) + [j0])))
+        x = g.standard_normal((n,) + dst.shape[1:], dtype=np.float32)
+        bf16_bits(x, out=dst[j0:j0 + n])
+
+    if len(chunks) <= 2:
+        for j0 in chunks:
+            work(j0)
+        return
+    with cf.ThreadPoolExecutor(max_workers=min(len(chunks), os.cpu_count() or 4)) as ex:
+        list(ex.map(work, chunks))
 
 
 def _model_widths(rng, spec: Spec, n_model: int):
@@ -344,13 +379,8 @@ def build(spec: Spec, seed: int = 0) -> Workload:
         rng = r["rng"]
         n0, N, S = int(node_off[b]), r["N"], r["S"]
         q[n0:n0 + N] = bf16_bits(rng.standard_normal((N, spec.Hq, spec.D), dtype=np.float32))
-        k0 = int(kv_off[b])
-        for dst in (k, v):
-            step = 4096
-            for j in range(0, S + N, step):
-                n = min(step, S + N - j)
-                dst[k0 + j:k0 + j + n] = bf16_bits(
-                    rng.standard_normal((n, spec.Hkv, spec.D), dtype=np.float32))
+        _fill_normal_bf16(k[int(kv_off[b]):int(kv_off[b]) + S + N], (seed, b, 0))
+        _fill_normal_bf16(v[int(kv_off[b]):int(kv_off[b]) + S + N], (seed, b, 1))
 
         # logits with planted acceptance structure
         z = rng.standard_normal((N, spec.V), dtype=np.float32)

@@ -1,0 +1,123 @@
+"""C-ABI library checks that need no GPU: it builds, loads, exports every
+symbol ``include/respec.h`` declares, and rejects bad host arguments before
+launching anything.  Also checks that the oracle and the CUDA library share
+no source."""
+import ctypes as C
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "respec.h")
+
+
+@pytest.fixture(scope="module")
+def rs():
+    from paper_2511_01282_gb300 import build
+    build.build()
+    from paper_2511_01282_gb300 import respec
+    respec.lib()
+    return respec
+
+
+def _declared():
+    txt = open(HEADER).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return sorted(set(re.findall(r"\b(rs_[a-z_]+)\s*\(", txt)))
+
+
+def test_header_declares_the_four_calls():
+    names = _declared()
+    for n in ("rs_entropy_gate", "rs_match_scan", "rs_tree_verify_attn", "rs_accept"):
+        assert n in names and n + "_workspace_size" in names
+
+
+def test_every_declared_symbol_is_exported(rs):
+    out = subprocess.run(["nm", "-D", "--defined-only", rs.LIB_PATH], capture_output=True, text=True,
+                         check=True).stdout
+    exported = set(re.findall(r"\bT (rs_\w+)", out))
+    missing = [n for n in _declared() if n not in exported]
+    assert not missing, missing
+    # and the binding knows each of them
+    assert sorted(rs.exported_symbols()) == sorted(_declared())
+
+
+def test_library_identifies_itself(rs):
+    assert "sm_103a" in rs.rs_version()
+    assert rs.rs_launch_count() >= 0
+
+
+def test_params_struct_layout_matches_header(rs):
+    # 11 four-byte fields, no padding
+    assert C.sizeof(rs.rs_params) == 44
+    txt = open(HEADER).read()
+    body = re.search(r"typedef struct \{(.*?)\} rs_params;", txt, re.S).group(1)
+    fields = re.findall(r"\b(int|float)\s+([a-z_]+)\s*;", re.sub(r"/\*.*?\*/", "", body, flags=re.S))
+    assert [f for _, f in fields] == [f for f, _ in rs.rs_params._fields_]
+
+
+def test_workspace_sizes_are_host_computable(rs):
+    assert rs.rs_entropy_gate_workspace_size(145, 128256) >= 145 * 16 * 12
+    assert rs.rs_accept_workspace_size(145, 128256, 5) >= 145 * 16 * 5 * 8
+    assert rs.rs_match_scan_workspace_size(4) >= 0
+    assert rs.rs_entropy_gate_workspace_size(-1, 10) == 0
+
+
+def _fake(n=1):
+    return C.c_void_p(0x10000)  # never dereferenced: every call below fails its host checks
+
+
+def test_bad_arguments_fail_before_launch(rs):
+    L = rs.lib()
+    p = rs.params()
+    f = _fake()
+    n_launch = rs.rs_launch_count()
+    # rs_entropy_gate: l out of range
+    bad = rs.params(l=0)
+    st = L.rs_entropy_gate(f, 1, 10, f, f, 1, bad, f, f, f, f, f, f, f, 1 << 20, None)
+    assert st == rs.RS_ERR_INVALID_ARG and "l=0" in rs.rs_last_error()
+    # V = 0
+    st = L.rs_entropy_gate(f, 1, 0, f, f, 1, p, f, f, f, f, f, f, f, 1 << 20, None)
+    assert st == rs.RS_ERR_INVALID_ARG
+    # workspace too small
+    st = L.rs_entropy_gate(f, 4, 100000, f, f, 1, p, f, f, f, f, f, f, f, 8, None)
+    assert st == rs.RS_ERR_CAPACITY and "workspace" in rs.rs_last_error()
+    # rs_accept: beta above V, negative tau, null pointers
+    st = L.rs_accept(f, 1, 3, f, 1, f, f, f, f, f, f, rs.params(beta=5), 4, *([f] * 11), f, 1 << 20, None)
+    assert st == rs.RS_ERR_INVALID_ARG
+    st = L.rs_accept(f, 1, 30, f, 1, f, f, f, f, f, f, rs.params(tau=-1.0), 4, *([f] * 11), f, 1 << 20, None)
+    assert st == rs.RS_ERR_INVALID_ARG
+    st = L.rs_accept(None, 1, 30, f, 1, f, f, f, f, f, f, p, 4, *([f] * 11), f, 1 << 20, None)
+    assert st == rs.RS_ERR_INVALID_ARG and "null" in rs.rs_last_error()
+    # rs_match_scan: top_c above the limit, span_len 0
+    st = L.rs_match_scan(f, f, 1, f, None, f, rs.params(top_c=9), 4, *([f] * 7), None, 0, None)
+    assert st == rs.RS_ERR_INVALID_ARG
+    st = L.rs_match_scan(f, f, 1, f, None, f, rs.params(span_len=0), 4, *([f] * 7), None, 0, None)
+    assert st == rs.RS_ERR_INVALID_ARG
+    # rs_tree_verify_attn: unsupported head dim, GQA mismatch, misaligned K
+    st = L.rs_tree_verify_attn(f, f, f, 10, f, f, f, f, 1, 1, 4, 4, 96, 0.1, f, f, f, f, 1 << 30, None)
+    assert st == rs.RS_ERR_UNSUPPORTED and "96" in rs.rs_last_error()
+    st = L.rs_tree_verify_attn(f, f, f, 10, f, f, f, f, 1, 1, 6, 4, 128, 0.1, f, f, f, f, 1 << 30, None)
+    assert st == rs.RS_ERR_UNSUPPORTED
+    st = L.rs_tree_verify_attn(f, C.c_void_p(0x10002), f, 10, f, f, f, f, 1, 1, 4, 4, 128, 0.1, f, f, f, f,
+                               1 << 30, None)
+    assert st == rs.RS_ERR_INVALID_ARG and "aligned" in rs.rs_last_error()
+    # nothing was launched by any of these
+    assert rs.rs_launch_count() == n_launch
+
+
+def test_oracle_and_library_share_no_source():
+    pkg = os.path.join(ROOT, "paper_2511_01282_gb300")
+    ora = os.path.join(ROOT, "oracle")
+    for d, other in ((pkg, "oracle"), (ora, "paper_2511_01282_gb300")):
+        for dirpath, _, files in os.walk(d):
+            for fn in files:
+                if fn.endswith((".c", ".h", ".cu", ".cuh", ".py")):
+                    txt = open(os.path.join(dirpath, fn)).read()
+                    assert not re.search(r"(import|include)[^\n]*\b%s\b" % other, txt), (fn, other)
+    # the oracle restates its own constants instead of including the ABI header
+    for fn in os.listdir(ora):
+        if fn.endswith((".c", ".h")):
+            assert "respec.h" not in open(os.path.join(ora, fn)).read()

@@ -1,0 +1,167 @@
+"""GPU edge cases: malformed and oversized trees, empty requests, unaligned
+and odd-sized logits, position-list truncation, skipped requests, and a
+CUDA-graph replay of the whole step."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from gpu_helpers import check_accept, check_gate, f32, host, make_step
+from paper_2511_01282_gb300 import respec as rs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def _cuda(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def _attn_inputs(rng, Hq, Hkv, D, S_list, trees):
+    node_off = np.concatenate([[0], np.cumsum([len(t) for t in trees])]).astype(np.int32)
+    sizes = [s + len(t) for s, t in zip(S_list, trees)]
+    kv_off = np.concatenate([[0], np.cumsum(sizes)[:-1]]).astype(np.int64)
+    T, R = int(sum(sizes)), int(node_off[-1])
+    q = synth.bf16_bits(rng.standard_normal((R, Hq, D)).astype(np.float32))
+    k = synth.bf16_bits(rng.standard_normal((max(T, 1), Hkv, D)).astype(np.float32))
+    v = synth.bf16_bits(rng.standard_normal((max(T, 1), Hkv, D)).astype(np.float32))
+    parents = np.concatenate([np.array(t, np.int32) for t in trees]) if R else np.zeros(0, np.int32)
+    return q, k, v, kv_off, np.array(S_list, np.int32), node_off, parents
+
+
+def _run_attn(q, k, v, kv_off, ctx, node_off, parents, Hq, Hkv, D, scale):
+    B, R = len(ctx), int(node_off[-1])
+    out = torch.full((max(R, 1), Hq, D), 7.0, device="cuda")
+    lse = torch.full((max(R, 1), Hq), 7.0, device="cuda")
+    status = torch.full((B,), -1, dtype=torch.int32, device="cuda")
+    ws = torch.empty(rs.rs_tree_verify_attn_workspace_size(B, R, Hq, Hkv, D), dtype=torch.uint8, device="cuda")
+    rs.rs_tree_verify_attn(_cuda(q), _cuda(k), _cuda(v), k.shape[0], _cuda(kv_off), _cuda(ctx), _cuda(node_off),
+                           _cuda(parents) if R else None, B, R, Hq, Hkv, D, scale, out, lse, status, ws)
+    torch.cuda.synchronize()
+    return host(out)[:R], host(lse)[:R], host(status)
+
+
+def test_attention_rejects_bad_trees_and_keeps_the_rest():
+    rng = np.random.default_rng(0)
+    Hq, Hkv, D = 4, 2, 128
+    good = [-1, 0, 0, 1, 3]
+    trees = [good, [-1, 0, 2, 1], [], [-1] + [int(rng.integers(0, i)) for i in range(1, 300)], good]
+    S = [130, 50, 10, 200, 0]
+    inp = _attn_inputs(rng, Hq, Hkv, D, S, trees)
+    out, lse, status = _run_attn(*inp, Hq, Hkv, D, D ** -0.5)
+    assert status.tolist() == [0, rs.RS_ST_BAD_TREE, 0, rs.RS_ST_TOO_LARGE, 0]
+    q, k, v, kv_off, ctx, node_off, parents = inp
+    for b in (1, 3):
+        n0, n1 = node_off[b], node_off[b + 1]
+        assert (out[n0:n1] == 0).all() and (lse[n0:n1] == 0).all()
+    for b in (0, 4):  # S = 0 for request 4: the tree alone
+        n0, n1 = int(node_off[b]), int(node_off[b + 1])
+        rows = [(n, h) for n in range(n0, n1) for h in range(Hq)]
+        ref = oracle.tree_attn(q, k, v, kv_off, ctx, node_off, parents, Hq, Hkv, D, D ** -0.5, rows=rows)
+        got = out[n0:n1].reshape(-1, D)
+        assert np.abs(got - ref["out"]).max() < 1e-2
+
+
+def test_attention_single_node_and_tile_straddling_tree():
+    rng = np.random.default_rng(1)
+    Hq, Hkv, D = 6, 3, 64
+    trees = [[-1], [-1] + list(range(0, 99)), [-1, 0, 1, 1, 0]]
+    S = [1, 90, 127]  # tree slots cross the 128-key tile boundary
+    inp = _attn_inputs(rng, Hq, Hkv, D, S, trees)
+    out, lse, status = _run_attn(*inp, Hq, Hkv, D, 0.3)
+    assert (status == 0).all()
+    q, k, v, kv_off, ctx, node_off, parents = inp
+    ref = oracle.tree_attn(q, k, v, kv_off, ctx, node_off, parents, Hq, Hkv, D, 0.3)
+    assert np.abs(out.reshape(-1, D) - ref["out"]).max() < 1e-2
+    assert np.abs(lse.reshape(-1) - ref["lse"]).max() < 1e-3
+
+
+def test_accept_rejects_bad_trees():
+    w = synth.build(synth.small_spec(B=4, V=700), seed=11)
+    # request 2: a model node hanging from a chain node
+    n0 = int(w.node_off[2])
+    src = w.source.copy()
+    ch = w.chain.copy()
+    src[n0 + 1], ch[n0 + 1] = 2, 0
+    w.source, w.chain = src, ch
+    st = make_step(w)
+    ref = check_accept(w, st)
+    assert ref["status"][2] & oracle.ST_BAD_TREE
+
+
+def test_unaligned_and_odd_logits():
+    w = synth.build(synth.small_spec(B=2, V=1003), seed=12)
+    st = make_step(w)
+    R, V = w.logits.shape
+    flat = torch.zeros(R * V + 1, dtype=torch.float32, device="cuda")
+    flat[1:] = torch.from_numpy(w.logits.reshape(-1)).cuda()
+    st.d["logits"] = flat[1:].view(R, V)  # 4-byte aligned only: scalar path
+    check_gate(w, st)
+    check_accept(w, st)
+
+
+def test_scan_truncation_and_skips():
+    w = synth.build(synth.small_spec(B=4, repeat_prob=0.9, seg_len=(2, 4), V=50), seed=13)
+    st = make_step(w)
+    st.pos_cap = 3
+    st.out["pos"] = torch.zeros((w.B, 3), dtype=torch.int32, device="cuda")
+    ks = np.array([1, 2, 9, 3], np.int32)          # 9 > RS_MAX_L: skipped with a status
+    ok = np.array([1, 1, 1, 0], np.uint8)          # request 3 not triggered
+    ks_o = ks.copy()
+    ks_o[2] = 0
+    # the oracle has no key-length cap: it sees the capped request as k = 0
+    st.scan(k_star=_cuda(ks), gate_ok=_cuda(ok))
+    torch.cuda.synchronize()
+    ref = oracle.match_scan(w.tokens, w.tok_off, ks_o, w.scores, f32(w.spec.theta_score), w.spec.top_c,
+                            w.spec.chain_len, 3, gate_ok=ok)
+    got_status = host(st.out["scan_status"])
+    assert got_status[2] == rs.RS_ST_TOO_LARGE
+    for key in ("count", "pos", "sel_pos", "sel_len", "spans", "n_sel"):
+        assert (host(st.out[key]) == ref[key]).all(), key
+    assert got_status[0] & rs.RS_ST_TRUNCATED and got_status[3] == 0
+    assert (ref["status"][[0, 1, 3]] == got_status[[0, 1, 3]]).all()
+
+
+def test_gate_with_empty_row_ranges():
+    w = synth.build(synth.small_spec(B=3, V=300), seed=14)
+    st = make_step(w)
+    # request 1 owns no rows this step: its history is only re-evaluated
+    off = w.node_off.copy()
+    off[2] = off[1]
+    st.d["row_off"] = _cuda(off.astype(np.int32))
+    st.gate()
+    torch.cuda.synchronize()
+    H = host(st.out["entropy"]).astype(np.float64)
+    g = oracle.gate(H, off, w.row_commit, w.hist, w.hist_n, w.spec.l, f32(w.spec.lambda_e),
+                    f32(w.spec.theta_entropy))
+    assert (host(st.out["k_star"]) == g["k_star"]).all()
+    assert (host(st.d["hist"]) == g["hist"].astype(np.float32)).all()
+
+
+def test_cuda_graph_replay_matches_eager():
+    w = synth.make("tiny")
+    st = make_step(w)
+    st.step()
+    torch.cuda.synchronize()
+    eager = {k: host(v).copy() for k, v in st.out.items()}
+    st.reset_state()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s):
+        st.step(stream=s)  # warm the stream once outside the capture
+    torch.cuda.synchronize()
+    st.reset_state()
+    with torch.cuda.graph(g, stream=s):
+        st.step(stream=s)
+    st.reset_state()
+    g.replay()
+    torch.cuda.synchronize()
+    for k, v in eager.items():
+        assert (host(st.out[k]) == v).all(), k
