@@ -255,8 +255,14 @@ def run_ours(args, rank, world, local_rank):
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph, stream=stream):
         st.step(stream)
+
+    def replay():
+        # a graph launches on the current stream: make that the timed stream
+        with torch.cuda.stream(stream):
+            graph.replay()
+
     for _ in range(max(W, 3)):
-        graph.replay()
+        replay()
     torch.cuda.synchronize()
 
     clocks = ClockSampler(local_rank)
@@ -274,7 +280,7 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize()
     e0.record(stream)
     for _ in range(K):
-        graph.replay()
+        replay()
     e1.record(stream)
     torch.cuda.synchronize()
     barrier()
@@ -305,7 +311,7 @@ def run_ours(args, rank, world, local_rank):
     bufs = st.result_buffers()
     for _ in range(max(W, 2)):
         st.upload(stream)
-        graph.replay()
+        replay()
         st.download_into(bufs, stream)
     torch.cuda.synchronize()
     barrier()
@@ -313,7 +319,7 @@ def run_ours(args, rank, world, local_rank):
     h2d = d2h = 0
     for _ in range(K):
         h2d = st.upload(stream)
-        graph.replay()
+        replay()
         d2h = st.download_into(bufs, stream)
         stream.synchronize()
     e2e_s = time.perf_counter() - t0

@@ -146,7 +146,9 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
     }
 }
 
-constexpr int kDecThreads = 256;
+constexpr int kDecThreads = 512;
+// candidates per lane when a warp merges one row: nchunks * beta <= 32 * 8
+constexpr int kCandPerLane = 8;
 
 __global__ void __launch_bounds__(kDecThreads)
 accept_decide(const float *__restrict__ logits, int V, int nchunks, const VI *__restrict__ cand,
@@ -177,7 +179,10 @@ accept_decide(const float *__restrict__ logits, int V, int nchunks, const VI *__
     __shared__ int s_bad;
     __shared__ int s_best;  // (depth << 16) | (0xffff - node)
 
-    // ---- row statistics (every row of the request) ----
+    // ---- row statistics (every row of the request): one warp per row ----
+    // the row's chunk candidates (<= 32 * kCandPerLane) are loaded once into
+    // registers, then beta rounds of a warp-wide "best after the previous
+    // winner" reduction run on them
     const int ncand = nchunks * beta;
     for (int lr = warp; lr < N; lr += kDecThreads / 32) {
         const long long r = n0 + lr;
@@ -188,30 +193,36 @@ accept_decide(const float *__restrict__ logits, int V, int nchunks, const VI *__
             MS u{__shfl_xor_sync(0xffffffffu, ms.m, o), __shfl_xor_sync(0xffffffffu, ms.s, o)};
             ms = ms_merge(ms, u);
         }
-        float l = ms.s > 0.f ? ms.m + __logf(ms.s) : -INFINITY;
+        const float l = ms.s > 0.f ? ms.m + __logf(ms.s) : -INFINITY;
+        VI cv[kCandPerLane];
+#pragma unroll
+        for (int q = 0; q < kCandPerLane; ++q) {
+            const int c = lane + 32 * q;
+            cv[q] = c < ncand ? cand[r * ncand + c] : VI{-INFINITY, kNoId};
+        }
         VI prev{INFINITY, -1};
         for (int k = 0; k < beta; ++k) {
             VI best{-INFINITY, kNoId};
-            for (int c = lane; c < ncand; c += 32) {
-                VI x = cand[r * ncand + c];
+#pragma unroll
+            for (int q = 0; q < kCandPerLane; ++q) {
+                const VI x = cv[q];
                 if (x.i != kNoId && vi_before(prev.v, prev.i, x.v, x.i) && vi_before(x.v, x.i, best.v, best.i))
                     best = x;
             }
             best = warp_vi_best(best);
             prev = best;
             if (lane == 0) {
-                int id = best.i == kNoId ? -1 : best.i;
+                const int id = best.i == kNoId ? -1 : best.i;
                 topk[r * beta + k] = id;
                 if (lr < RS_MAX_NODES) s_top[lr * RS_MAX_BETA + k] = id;
-            }
-        }
-        if (lane == 0) {
-            int a0 = topk[r * beta];
-            argmax[r] = a0;
-            lse[r] = l;
-            if (lr < RS_MAX_NODES) {
-                s_arg[lr] = a0;
-                s_lse[lr] = l;
+                if (k == 0) {
+                    argmax[r] = id;
+                    lse[r] = l;
+                    if (lr < RS_MAX_NODES) {
+                        s_arg[lr] = id;
+                        s_lse[lr] = l;
+                    }
+                }
             }
         }
     }
@@ -423,6 +434,11 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
                             scores && status),
                  "rs_accept: null request pointer");
     const int nchunks = (V + kAccChunk - 1) / kAccChunk;
+    if (nchunks * p.beta > 32 * kCandPerLane) {
+        set_error("rs_accept: V=%d with beta=%d exceeds the %d top-k candidates a row merge holds", V, p.beta,
+                  32 * kCandPerLane);
+        return RS_ERR_UNSUPPORTED;
+    }
     const size_t need = rs_accept_workspace_size(R, V, p.beta);
     if (workspace_bytes < need || (need && !workspace)) {
         set_error("rs_accept: workspace %zu bytes < %zu required", workspace_bytes, need);

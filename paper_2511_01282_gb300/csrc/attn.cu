@@ -1,34 +1,32 @@
 // attn.cu -- rs_tree_verify_attn: attention of the verify pass over the
 // packed draft tree (Algorithm 1 l.13 / l.25; "parallel verification" of
-// Section 3.3).  Node i of request b attends to the b's committed prefix and
-// to the tree slots of its ancestors and itself.
+// Section 3.3).  Node i of request b attends to b's committed prefix and to
+// the tree slots of its ancestors and itself.
 //
-// Work decomposition (identical for every compute core):
+// Work decomposition:
 //   segment = (request b, KV head, row tile of 128 (node, q-head-in-group)
 //             rows); unit = one 128-key KV tile of a segment.
-//   The units of all segments are laid end to end and cut into gridDim.x
-//   equal ranges, one per CTA, so every SM streams the same number of KV
-//   tiles whatever the mix of context lengths (a stream-K split).  A segment
-//   that lies inside one CTA's range is finished by that CTA; a segment cut
-//   by range boundaries leaves one partial (unnormalised O, running max,
-//   running sum) per piece, in one of two slots per CTA, and the combine
-//   kernel merges them.  Nothing spins or waits across CTAs.
+//   The units of all segments are laid end to end and cut into one equal
+//   range per SM, so every SM streams the same number of KV tiles whatever
+//   the mix of context lengths (a stream-K split).  A segment that lies
+//   inside one CTA's range is finished by that CTA; a segment cut by range
+//   boundaries leaves one partial (unnormalised O, running max, running sum)
+//   per piece, in one of two slots per CTA, and attn_combine merges them.
+//   Nothing spins or waits across CTAs.
 //   attn_prep validates each tree and builds a 256-bit ancestor set per
 //   node; the tree part of the mask is a bit test on it.
+// Launches: attn_prep (B CTAs) -> attn_tc_kernel (one CTA per SM; see
+// attn_core.cuh) -> attn_combine (one CTA per SM).
+#include <cudaTypedefs.h>
 #include <math.h>
+
+#include <mutex>
 
 #include "attn_core.cuh"
 #include "common.cuh"
 
 namespace rs {
 namespace {
-
-struct ReqInfo {
-    int units;  // Hkv * mt * nt, 0 for a rejected request
-    int mt;     // row tiles
-    int nt;     // KV tiles
-    int ok;
-};
 
 __global__ void __launch_bounds__(256)
 attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_len,
@@ -62,7 +60,7 @@ attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_
             uint32_t bits[kAncWords];
 #pragma unroll
             for (int w = 0; w < kAncWords; ++w) bits[w] = 0;
-            for (int a = i; a >= 0; a = s_par[a]) bits[a >> 5] |= 1u << (a & 31);
+            for (int x = i; x >= 0; x = s_par[x]) bits[x >> 5] |= 1u << (x & 31);
 #pragma unroll
             for (int w = 0; w < kAncWords; ++w) anc[(long long)(n0 + i) * kAncWords + w] = bits[w];
         }
@@ -82,93 +80,7 @@ attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_
     if (tid == 0) status[b] = st;
 }
 
-// Exclusive prefix of per-request units into s_pref[0..B] (s_pref[B] = W).
-__device__ void unit_prefix(const ReqInfo *__restrict__ info, int B, int *s_pref) {
-    __shared__ int s_carry;
-    if (threadIdx.x == 0) s_carry = 0;
-    __syncthreads();
-    for (int base = 0; base < B; base += blockDim.x) {
-        int i = base + threadIdx.x;
-        int v = i < B ? info[i].units : 0;
-        // inclusive warp scan, then across warps (blockDim.x <= 1024)
-        __shared__ int s_w[32];
-        int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-        int x = v;
-        for (int o = 1; o < 32; o <<= 1) {
-            int y = __shfl_up_sync(0xffffffffu, x, o);
-            if (lane >= o) x += y;
-        }
-        if (lane == 31) s_w[warp] = x;
-        __syncthreads();
-        if (warp == 0) {
-            int nw = (blockDim.x + 31) >> 5;
-            int w = lane < nw ? s_w[lane] : 0;
-            int z = w;
-            for (int o = 1; o < 32; o <<= 1) {
-                int y = __shfl_up_sync(0xffffffffu, z, o);
-                if (lane >= o) z += y;
-            }
-            s_w[lane] = z - w;
-        }
-        __syncthreads();
-        int incl = s_carry + s_w[warp] + x;
-        if (i < B) s_pref[i + 1] = incl;
-        __syncthreads();
-        if (threadIdx.x == blockDim.x - 1) s_carry = incl;
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) s_pref[0] = 0;
-    __syncthreads();
-}
-
-// last b with s_pref[b] <= u (requests with no units are skipped)
-__device__ __forceinline__ int find_req(const int *s_pref, int B, long long u) {
-    int lo = 0, hi = B - 1;
-    while (lo < hi) {
-        int mid = (lo + hi + 1) >> 1;
-        if (s_pref[mid] <= u) lo = mid;
-        else hi = mid - 1;
-    }
-    while (lo + 1 <= B - 1 && s_pref[lo + 1] <= u) ++lo;
-    return lo;
-}
-
-__device__ __forceinline__ long long range_lo(long long c, long long W, long long G) { return c * W / G; }
-__device__ __forceinline__ long long owner_of(long long u, long long W, long long G) {
-    return ((u + 1) * G - 1) / W;
-}
-
-__global__ void __launch_bounds__(kAttnThreads)
-attn_main(AttnArgs a, const ReqInfo *__restrict__ info) {
-    extern __shared__ __align__(1024) unsigned char smem[];
-    int *s_pref = reinterpret_cast<int *>(smem + kAttnSmemTiles);
-    unit_prefix(info, a.B, s_pref);
-    const long long W = s_pref[a.B];
-    const long long Gc = gridDim.x, c = blockIdx.x;
-    const long long u0 = range_lo(c, W, Gc), u1 = range_lo(c + 1, W, Gc);
-    long long u = u0;
-    while (u < u1) {
-        const int b = find_req(s_pref, a.B, u);
-        const ReqInfo ri = info[b];
-        const long long local = u - s_pref[b];
-        const int seg = (int)(local / ri.nt);
-        const int j0 = (int)(local - (long long)seg * ri.nt);
-        const long long seg_start = s_pref[b] + (long long)seg * ri.nt;
-        const long long seg_end = seg_start + ri.nt;
-        const long long pend = seg_end < u1 ? seg_end : u1;
-        Piece pc;
-        pc.b = b;
-        pc.kvh = seg / ri.mt;
-        pc.mtile = seg - pc.kvh * ri.mt;
-        pc.j0 = j0;
-        pc.j1 = j0 + (int)(pend - u);
-        pc.final = (seg_start >= u0 && seg_end <= u1);
-        pc.slot = (int)(2 * c + (seg_start > u0 ? 1 : 0));
-        attn_piece(a, pc, smem);
-        u = pend;
-    }
-}
-
+// Block c merges the split segment whose first piece is c's last piece.
 __global__ void __launch_bounds__(256)
 attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
     extern __shared__ int s_pref[];
@@ -220,14 +132,43 @@ attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
     }
 }
 
-int g_attr_done[64] = {0};
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static std::once_flag once;
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// [kv_rows, Hkv, D] bf16 viewed as a 3-D tensor (D, Hkv, kv_rows); boxes of
+// 64 head-dim columns x 1 head x 128 keys, 128-byte swizzled, zero fill.
+bool make_kv_map(CUtensorMap *m, const void *base, long long kv_rows, int Hkv, int D) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)Hkv, (cuuint64_t)kv_rows};
+    cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)Hkv * D * 2};
+    cuuint32_t box[3] = {64, 1, (cuuint32_t)kBN};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+int g_attr_done[64][2] = {};
 
 }  // namespace
 }  // namespace rs
 
 using namespace rs;
 
-static int attn_grid() { return num_sms() * kAttnCtasPerSm; }
+static int attn_grid() { return num_sms(); }
 
 extern "C" size_t rs_tree_verify_attn_workspace_size(int B, int R, int Hq, int Hkv, int D) {
     if (B < 0 || R < 0 || Hq < 1 || Hkv < 1 || (D != 64 && D != 128)) return 0;
@@ -256,7 +197,8 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
         set_error("rs_tree_verify_attn: Hq=%d must be a positive multiple of Hkv=%d", Hq, Hkv);
         return RS_ERR_UNSUPPORTED;
     }
-    RS_CHECK_ARG(B <= 16384, "rs_tree_verify_attn: B=%d above 16384", B);
+    RS_CHECK_ARG(B <= kAttnMaxB, "rs_tree_verify_attn: B=%d above %d", B, kAttnMaxB);
+    RS_CHECK_ARG(kv_rows < (1ll << 31) - kBN, "rs_tree_verify_attn: kv_rows above 2^31");
     RS_CHECK_ARG(isfinite(scale), "rs_tree_verify_attn: scale must be finite");
     RS_CHECK_ARG(B == 0 || (kv_off && ctx_len && node_off && status), "rs_tree_verify_attn: null request pointer");
     RS_CHECK_ARG(R == 0 || (q && parents && out && lse), "rs_tree_verify_attn: null row pointer");
@@ -275,8 +217,6 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     uint32_t *anc = cv.take<uint32_t>((size_t)R * kAncWords);
     AttnArgs a;
     a.q = q;
-    a.k = k;
-    a.v = v;
     a.kv_off = kv_off;
     a.ctx_len = ctx_len;
     a.node_off = node_off;
@@ -291,24 +231,41 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     a.scale = scale;
     a.out = out;
     a.lse = lse;
+    a.status = status;
     cudaStream_t st = (cudaStream_t)stream;
+
+    // a map over an empty KV cache is never dereferenced: point it at q
+    CUtensorMap tmk, tmv;
+    const long long rows_map = kv_rows > 0 ? kv_rows : 1;
+    if (!make_kv_map(&tmk, kv_rows > 0 ? (const void *)k : (const void *)q, rows_map, Hkv, D) ||
+        !make_kv_map(&tmv, kv_rows > 0 ? (const void *)v : (const void *)q, rows_map, Hkv, D)) {
+        set_error("rs_tree_verify_attn: cuTensorMapEncodeTiled failed");
+        return RS_ERR_CUDA;
+    }
 
     attn_prep<<<B, 256, 0, st>>>(node_off, ctx_len, parents, Hq, Hkv, D, info, anc, out, lse, status);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/prep");
 
-    const size_t smem_main = kAttnSmemTiles + (size_t)(B + 1) * sizeof(int);
     int dev = 0;
     cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !g_attr_done[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(attn_main, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             kAttnSmemTiles + (16384 + 1) * (int)sizeof(int));
+    const int di = D == 128 ? 1 : 0;
+    const size_t smem_max = attn_smem_bytes(kAttnMaxB);
+    if (dev >= 0 && dev < 64 && !g_attr_done[dev][di]) {
+        cudaError_t e = D == 128 ? cudaFuncSetAttribute(attn_tc_kernel<128>,
+                                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_max)
+                                 : cudaFuncSetAttribute(attn_tc_kernel<64>,
+                                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_max);
         if (e != cudaSuccess) {
             set_error("rs_tree_verify_attn: cudaFuncSetAttribute: %s", cudaGetErrorString(e));
             return RS_ERR_CUDA;
         }
-        g_attr_done[dev] = 1;
+        g_attr_done[dev][di] = 1;
     }
-    attn_main<<<Gc, kAttnThreads, smem_main, st>>>(a, info);
+    const size_t smem = attn_smem_bytes(B);
+    if (D == 128)
+        attn_tc_kernel<128><<<Gc, kAttnThreads, smem, st>>>(a, info, tmk, tmv);
+    else
+        attn_tc_kernel<64><<<Gc, kAttnThreads, smem, st>>>(a, info, tmk, tmv);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/main");
     attn_combine<<<Gc, 256, (size_t)(B + 1) * sizeof(int), st>>>(a, info);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/combine");

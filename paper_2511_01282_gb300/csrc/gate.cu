@@ -114,6 +114,8 @@ entropy_partial(const float *__restrict__ logits, int V, int nchunks, Ent3 *__re
     }
 }
 
+constexpr int kFinRows = 512;  // rows staged in shared memory per pass
+
 __global__ void __launch_bounds__(256)
 gate_finalize(const Ent3 *__restrict__ part, int nchunks, const int32_t *__restrict__ row_off,
               const uint8_t *__restrict__ row_commit, rs_params p, float *__restrict__ hist,
@@ -122,34 +124,52 @@ gate_finalize(const Ent3 *__restrict__ part, int nchunks, const int32_t *__restr
     const int b = blockIdx.x;
     const int r0 = row_off[b], r1 = row_off[b + 1];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-
-    // row entropies: one warp per row, lanes over chunks
-    for (int r = r0 + warp; r < r1; r += blockDim.x >> 5) {
-        Ent3 t{-INFINITY, 0.f, 0.f};
-        for (int c = lane; c < nchunks; c += 32) t = ent_merge(t, part[(long long)r * nchunks + c]);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) t = ent_merge(t, ent_shfl(t, o));
-        if (lane == 0) entropy[r] = t.s > 0.f ? (__logf(t.s) - t.w / t.s) : 0.f;
-    }
-    __syncthreads();  // this block's entropy[] writes are visible below
-
-    if (threadIdx.x != 0) return;
+    __shared__ float s_ent[kFinRows];
+    __shared__ uint8_t s_com[kFinRows];
+    __shared__ float s_h[RS_MAX_L];
+    __shared__ int s_n;
     const int l = p.l;
-    float h[RS_MAX_L];
-    int n = hist_n[b];
-    n = n < 0 ? 0 : (n > l ? l : n);
-    for (int i = 0; i < l; ++i) h[i] = hist[(long long)b * l + i];
-    for (int r = r0; r < r1; ++r) {
-        if (!row_commit[r]) continue;
-        float e = entropy[r];
-        if (n == l) {
-            for (int i = 1; i < l; ++i) h[i - 1] = h[i];
-            h[l - 1] = e;
-        } else {
-            h[n++] = e;
-        }
+    if (threadIdx.x == 0) {
+        int n = hist_n[b];
+        n = n < 0 ? 0 : (n > l ? l : n);
+        s_n = n;
+        for (int i = 0; i < l; ++i) s_h[i] = hist[(long long)b * l + i];
     }
-    for (int i = 0; i < l; ++i) hist[(long long)b * l + i] = h[i];
+    for (int base = r0; base < r1; base += kFinRows) {
+        const int rows = min(kFinRows, r1 - base);
+        // row entropies: one warp per row, lanes over chunks
+        for (int lr = warp; lr < rows; lr += blockDim.x >> 5) {
+            const long long r = base + lr;
+            Ent3 t{-INFINITY, 0.f, 0.f};
+            for (int c = lane; c < nchunks; c += 32) t = ent_merge(t, part[r * nchunks + c]);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) t = ent_merge(t, ent_shfl(t, o));
+            if (lane == 0) {
+                const float e = t.s > 0.f ? (__logf(t.s) - t.w / t.s) : 0.f;
+                entropy[r] = e;
+                s_ent[lr] = e;
+            }
+        }
+        for (int lr = threadIdx.x; lr < rows; lr += blockDim.x) s_com[lr] = row_commit[base + lr];
+        __syncthreads();
+        if (threadIdx.x == 0) {  // push the committed rows, in row order
+            int n = s_n;
+            for (int lr = 0; lr < rows; ++lr) {
+                if (!s_com[lr]) continue;
+                if (n == l) {
+                    for (int i = 1; i < l; ++i) s_h[i - 1] = s_h[i];
+                    s_h[l - 1] = s_ent[lr];
+                } else {
+                    s_h[n++] = s_ent[lr];
+                }
+            }
+            s_n = n;
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x != 0) return;
+    const int n = s_n;
+    for (int i = 0; i < l; ++i) hist[(long long)b * l + i] = s_h[i];
     hist_n[b] = n;
 
     // Algorithm 1 step 1 in fp64: k upward, strict '<'
@@ -157,7 +177,7 @@ gate_finalize(const Ent3 *__restrict__ part, int nchunks, const int32_t *__restr
     int kbest = 0;
     for (int k = 1; k <= n; ++k) {
         double s = 0.0;
-        for (int i = n - k; i < n; ++i) s = __dadd_rn(s, (double)h[i]);
+        for (int i = n - k; i < n; ++i) s = __dadd_rn(s, (double)s_h[i]);
         double hk = __ddiv_rn(s, (double)k);
         double ck = __dadd_rn(hk, __ddiv_rn((double)p.lambda_e, (double)k));
         if (ck < c_min) {
