@@ -64,6 +64,8 @@ typedef enum {
 #define RS_ST_TRUNCATED  2  /* an output list was longer than its capacity     */
 #define RS_ST_BAD_POS    4  /* a selected position lies outside the buffer     */
 #define RS_ST_TOO_LARGE  8  /* more than RS_MAX_NODES tree nodes               */
+#define RS_ST_TIMEOUT   16  /* a pipeline wait inside a kernel gave up (bounded
+                               wait, ~2 s); the request's outputs are invalid   */
 
 /* -------------------------------------------------------------- parameters */
 /* Hyper-parameters of Algorithm 1 (Require line), Eq. 6-7 and Section 3.4.

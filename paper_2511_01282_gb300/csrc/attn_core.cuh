@@ -45,7 +45,6 @@ constexpr int kSmemPref = kSmemMisc + 16;
 constexpr int kAttnMaxB = 8192;
 constexpr long long kWaitLimit = 4000000000ll;     // clock cycles (~2 s)
 constexpr uint32_t kTmemCols = 512;
-constexpr int RS_ST_TIMEOUT_BIT = 16;
 
 inline size_t attn_smem_bytes(int B) { return 1024 + kSmemPref + (size_t)(B + 1) * sizeof(int); }
 
@@ -474,7 +473,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
         if (!ok && r == 0) {
             for (long long u = u0; u < u1;) {  // flag every request this CTA touches
                 const Piece pc = piece_at(info, s_pref, a.B, u, u0, u1, c);
-                atomicOr(&a.status[pc.b], RS_ST_TIMEOUT_BIT);
+                atomicOr(&a.status[pc.b], RS_ST_TIMEOUT);
                 u = pc.end;
             }
         }
