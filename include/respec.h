@@ -126,6 +126,31 @@ rs_status rs_entropy_gate(const float *logits, int R, int V, const int32_t *row_
                           int32_t *k_star, float *h_best, uint8_t *entropy_ok,
                           void *workspace, size_t workspace_bytes, void *stream);
 
+/* ============================================= rs_entropy_gate_noalloc ====
+ * Not from the paper (it has no counterpart): rs_entropy_gate for callers
+ * that cannot allocate device memory -- for example code embedded in a
+ * serving engine whose memory pool owns all of the GPU's memory and hands out
+ * no scratch buffers, or code that must not call cudaMalloc because that
+ * would synchronise the device in the middle of its work.  The caller still
+ * passes every input and output (same meaning as rs_entropy_gate); the
+ * library's scratch is a fixed device array of RS_GATE_NOALLOC_MAX_PARTIALS
+ * (max, sum, weighted-sum) triples (768 KiB) that every GPU loading the
+ * library holds until the process exits.  It supports
+ * R * ceil(V / 8192) <= RS_GATE_NOALLOC_MAX_PARTIALS (e.g. R <= 4096 rows at
+ * V = 128256); larger calls return RS_ERR_CAPACITY without launching.
+ * The first call on each device looks the array's device address up
+ * (cudaGetSymbolAddress), so make that first call before any stream capture.
+ * Nothing in the array needs to start at zero.  All calls share the array:
+ * calls that overlap on the GPU (other streams, or unordered host threads)
+ * race on it.  This call allocates nothing.
+ */
+#define RS_GATE_NOALLOC_MAX_PARTIALS 65536
+rs_status rs_entropy_gate_noalloc(const float *logits, int R, int V, const int32_t *row_off,
+                                  const uint8_t *row_commit, int B, rs_params p,
+                                  float *hist, int32_t *hist_n, float *entropy,
+                                  int32_t *k_star, float *h_best, uint8_t *entropy_ok,
+                                  void *stream);
+
 /* ======================================================= rs_match_scan ====
  * Section 3.3 "Selection Algorithm" and Algorithm 1 l.9-11: find every
  * earlier occurrence of the key (the buffer's last k = k_star[b] tokens),

@@ -12,6 +12,8 @@
 // history and evaluates H_k, C_k, k* and the trigger in fp64.
 #include <math.h>
 
+#include <mutex>
+
 #include "common.cuh"
 
 namespace rs {
@@ -240,6 +242,84 @@ extern "C" rs_status rs_entropy_gate(const float *logits, int R, int V, const in
         gate_finalize<<<B, 256, 0, st>>>(part, nchunks, row_off, row_commit, p, hist, hist_n, entropy,
                                          k_star, h_best, entropy_ok);
         RS_CHECK_LAUNCH("rs_entropy_gate/gate_finalize");
+    }
+    return RS_OK;
+}
+
+// ============================================================ no-allocation variant
+// rs_entropy_gate_noalloc runs the same two kernels as rs_entropy_gate, with
+// the per-chunk partials in the fixed device array below instead of a caller
+// workspace, for callers that cannot allocate device memory.  The array
+// (RS_GATE_NOALLOC_MAX_PARTIALS triples, 12 bytes each) lives on every GPU that
+// loads this library until the process exits.  It needs no initialisation:
+// every partial a call reads was written earlier by the same call.  All calls
+// share it, so calls that overlap on the GPU (different streams, or several
+// host threads without ordering) race on it.
+static __device__ __align__(256) Ent3 g_gate_scratch[RS_GATE_NOALLOC_MAX_PARTIALS];
+
+// Device address of g_gate_scratch on the current device, looked up once per
+// device (the host-side name is only a stand-in for the symbol).
+static Ent3 *gate_scratch_address(int dev) {
+    static std::mutex mu;
+    static Ent3 *addr[64] = {nullptr};
+    if (dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lk(mu);
+    if (!addr[dev]) {
+        void *ptr = nullptr;
+        cudaError_t e = cudaGetSymbolAddress(&ptr, g_gate_scratch);
+        if (e != cudaSuccess) {
+            set_error("rs_entropy_gate_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+            return nullptr;
+        }
+        addr[dev] = static_cast<Ent3 *>(ptr);
+    }
+    return addr[dev];
+}
+
+extern "C" rs_status rs_entropy_gate_noalloc(const float *logits, int R, int V, const int32_t *row_off,
+                                             const uint8_t *row_commit, int B, rs_params p, float *hist,
+                                             int32_t *hist_n, float *entropy, int32_t *k_star, float *h_best,
+                                             uint8_t *entropy_ok, void *stream) {
+    clear_error();
+    RS_CHECK_ARG(R >= 0 && B >= 0, "rs_entropy_gate_noalloc: negative size (R=%d, B=%d)", R, B);
+    RS_CHECK_ARG(V >= 1, "rs_entropy_gate_noalloc: V must be >= 1 (got %d)", V);
+    RS_CHECK_ARG(p.l >= 1 && p.l <= RS_MAX_L, "rs_entropy_gate_noalloc: l=%d outside [1, %d]", p.l, RS_MAX_L);
+    RS_CHECK_ARG(R == 0 || (logits && entropy && row_commit), "rs_entropy_gate_noalloc: null row pointer");
+    RS_CHECK_ARG(B == 0 || (row_off && hist && hist_n && k_star && h_best && entropy_ok),
+                 "rs_entropy_gate_noalloc: null request pointer");
+    const int nchunks = (V + kGateChunk - 1) / kGateChunk;
+    const long long partials = (long long)R * nchunks;
+    if (partials > RS_GATE_NOALLOC_MAX_PARTIALS) {
+        set_error("rs_entropy_gate_noalloc: R=%d rows x %d chunks of %d logits = %lld partials exceed the "
+                  "fixed scratch of %d (at most %d rows at this V)",
+                  R, nchunks, kGateChunk, partials, RS_GATE_NOALLOC_MAX_PARTIALS,
+                  RS_GATE_NOALLOC_MAX_PARTIALS / nchunks);
+        return RS_ERR_CAPACITY;
+    }
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) {
+        set_error("rs_entropy_gate_noalloc: cudaGetDevice: %s", cudaGetErrorString(e));
+        return RS_ERR_CUDA;
+    }
+    Ent3 *part = gate_scratch_address(dev);
+    if (!part) {
+        if (!rs_last_error()[0]) set_error("rs_entropy_gate_noalloc: device %d not supported", dev);
+        return RS_ERR_CUDA;
+    }
+    cudaStream_t st = (cudaStream_t)stream;
+    if (R > 0) {
+        bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
+        if (vec)
+            entropy_partial<true><<<(unsigned)partials, kGateThreads, 0, st>>>(logits, V, nchunks, part);
+        else
+            entropy_partial<false><<<(unsigned)partials, kGateThreads, 0, st>>>(logits, V, nchunks, part);
+        RS_CHECK_LAUNCH("rs_entropy_gate_noalloc/entropy_partial");
+    }
+    if (B > 0) {
+        gate_finalize<<<B, 256, 0, st>>>(part, nchunks, row_off, row_commit, p, hist, hist_n, entropy, k_star,
+                                         h_best, entropy_ok);
+        RS_CHECK_LAUNCH("rs_entropy_gate_noalloc/gate_finalize");
     }
     return RS_OK;
 }

@@ -52,6 +52,8 @@ _SIGS = {
     "rs_entropy_gate_workspace_size": (C.c_size_t, [C.c_int, C.c_int]),
     "rs_entropy_gate": (C.c_int, [_P, C.c_int, C.c_int, _P, _P, C.c_int, rs_params,
                                   _P, _P, _P, _P, _P, _P, _P, C.c_size_t, _P]),
+    "rs_entropy_gate_noalloc": (C.c_int, [_P, C.c_int, C.c_int, _P, _P, C.c_int, rs_params,
+                                          _P, _P, _P, _P, _P, _P, _P]),
     "rs_match_scan_workspace_size": (C.c_size_t, [C.c_int]),
     "rs_match_scan": (C.c_int, [_P, _P, C.c_int, _P, _P, _P, rs_params, C.c_int,
                                 _P, _P, _P, _P, _P, _P, _P, _P, C.c_size_t, _P]),
@@ -140,6 +142,18 @@ def rs_entropy_gate(logits, R, V, row_off, row_commit, B, p, hist, hist_n, entro
     _check(lib().rs_entropy_gate(_ptr(logits), R, V, _ptr(row_off), _ptr(row_commit), B, p,
                                  _ptr(hist), _ptr(hist_n), _ptr(entropy), _ptr(k_star),
                                  _ptr(h_best), _ptr(entropy_ok), wp, wb, _stream(stream)))
+
+
+RS_GATE_NOALLOC_MAX_PARTIALS = 65536
+
+
+def rs_entropy_gate_noalloc(logits, R, V, row_off, row_commit, B, p, hist, hist_n, entropy, k_star,
+                            h_best, entropy_ok, stream=None):
+    """rs_entropy_gate with the library's fixed scratch array instead of a
+    caller workspace (for callers that cannot allocate device memory)."""
+    _check(lib().rs_entropy_gate_noalloc(_ptr(logits), R, V, _ptr(row_off), _ptr(row_commit), B, p,
+                                         _ptr(hist), _ptr(hist_n), _ptr(entropy), _ptr(k_star),
+                                         _ptr(h_best), _ptr(entropy_ok), _stream(stream)))
 
 
 def rs_match_scan_workspace_size(B):
