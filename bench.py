@@ -49,6 +49,8 @@ def parse():
     ap.add_argument("--cpu-budget-s", type=float, default=12.0,
                     help="seconds of oracle attention work in the CPU baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--requests", type=int, default=0,
+                    help="keep only the first N requests of the workload (small profiling cases)")
     return ap.parse_args()
 
 
@@ -235,7 +237,11 @@ def run_ours(args, rank, world, local_rank):
     dist = None
     if world > 1:
         import torch.distributed as dist
-    w = synth.build(synth.CONFIGS[args.workload], seed=args.seed + 7919 * rank)
+    spec = synth.CONFIGS[args.workload]
+    if args.requests:
+        import dataclasses
+        spec = dataclasses.replace(spec, B=min(args.requests, spec.B))
+    w = synth.build(spec, seed=args.seed + 7919 * rank)
     s = w.spec
     p = rs.params(**s.params())
     st = VerifyStep(arrays_from_workload(w), p, s.Hq, s.Hkv, s.D, pos_cap=s.pos_cap, pinned_host=True)
@@ -292,20 +298,27 @@ def run_ours(args, rank, world, local_rank):
     ms_per_step = t_ms / K
     value = K * world / (t_ms / 1e3)
 
-    # ---- per-call device time (events on the launching stream)
+    # ---- per-call device time: a CUDA graph of n back-to-back calls, replayed
+    # on the timed stream between two events (no host launch gaps inside)
     def time_call(fn, n):
-        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
-        for a, b in evs:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for _ in range(n):
+                fn(stream)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            g.replay()  # warm
             a.record(stream)
-            fn(stream)
+            g.replay()
             b.record(stream)
         torch.cuda.synchronize()
-        return statistics.mean(a.elapsed_time(b) for a, b in evs)
+        return a.elapsed_time(b) / n
 
-    n_call = max(5, min(K, 50))
-    st.reset_state()
+    n_call = max(5, min(K, 20))
     call_ms = {"gate": time_call(st.gate, n_call), "scan": time_call(lambda sm: st.scan(stream=sm), n_call),
                "attn": time_call(st.attn, n_call), "accept": time_call(lambda sm: st.accept(stream=sm), n_call)}
+    st.reset_state()
+    torch.cuda.synchronize()
 
     # ---- end to end: pinned host inputs -> step -> decisions back to the host
     bufs = st.result_buffers()
@@ -340,7 +353,8 @@ def run_ours(args, rank, world, local_rank):
         "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": K, "warmup": W,
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16+f32", "data": "synthetic",
-        "config": {"workload": WORKLOAD_TEXT[args.workload], "name": args.workload, "batch_per_gpu": s.B,
+        "config": {"workload": WORKLOAD_TEXT[args.workload] + (" (first %d requests)" % s.B if args.requests else ""),
+                   "name": args.workload, "batch_per_gpu": s.B,
                    "l2": "no flush: every step streams %.2f GB of KV + logits, > 129 MB L2"
                          % ((by["kv"] + 2 * by["logits"]) / 1e9),
                    "graph": "each step replays one CUDA graph of the 4 calls"},

@@ -200,11 +200,12 @@ rs_status rs_match_scan(const int32_t *tokens, const int64_t *tok_off, int B,
  *   k, v     [kv_rows, Hkv, D] bf16 KV cache; request b's prefix slot j
  *            (j < ctx_len[b]) is row kv_off[b] + j and its tree node i is row
  *            kv_off[b] + ctx_len[b] + i.  k and v must be 16-byte aligned.
- *   kv_off   [B] int64;  ctx_len [B] int32 (>= 0);  node_off [B+1] int32.
+ *   kv_off   [B] int64;  ctx_len [B] int32 (>= 0);  node_off [B+1] int32;
+ *            B <= 4096 requests per call; kv_rows < 2^31.
  *   parents  [R] int32 local parent index per node; parents of node 0 is -1,
  *            0 <= parents[i] < i otherwise.
  *   D in {64, 128}; Hq a multiple of Hkv (grouped-query heads h share KV
- *   head h / (Hq / Hkv)); scale is the softmax scale (1/sqrt(D) usually).
+ *   head h / (Hq / Hkv)); scale > 0 is the softmax scale (1/sqrt(D) usually).
  *   out      [R, Hq, D] fp32 attention outputs;  lse [R, Hq] fp32 natural-log
  *            sum of exp(scale * q.k) over the attended keys.
  *   status   [B]: RS_ST_BAD_TREE / RS_ST_TOO_LARGE for a malformed request

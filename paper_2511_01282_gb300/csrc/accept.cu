@@ -4,9 +4,13 @@
 //
 // Kernel 1 (accept_rows): one CTA per (row, 8192-logit chunk).  Each thread
 // holds 32 logits in registers; the CTA produces the chunk's (max, sum e^(z -
-// max)) pair and its beta best (logit, id) pairs, found by beta rounds of a
-// block-wide "best after the previous winner" reduction in the total order
-// (logit desc, id asc) -- no sorting, no dynamic register indexing.
+// max)) pair and its beta best (logit, id) pairs in the total order (logit
+// desc, id asc).  Each warp first bounds its beta-th largest logit from below
+// by the beta-th largest of its 32 lane maxima (a warp bitonic sort), appends
+// the few logits at or above that bound to shared memory and ranks only those
+// by beta rounds of a "best after the previous winner" warp reduction (exact;
+// with many ties at the bound it ranks all of the warp's logits instead);
+// warp 0 merges the eight lists.  No dynamic register indexing.
 // Kernel 2 (accept_decide): one CTA per request.  Warps merge the chunk
 // candidates of each row (argmax, top-beta, lse); then the block checks the
 // tree, verifies model nodes (each thread walks its own root path), runs the
@@ -15,6 +19,7 @@
 #include <math.h>
 
 #include "common.cuh"
+#include "sm100.cuh"
 
 namespace rs {
 namespace {
@@ -23,6 +28,7 @@ constexpr int kAccThreads = 256;
 constexpr int kAccVpt = 32;
 constexpr int kAccChunk = kAccThreads * kAccVpt;
 constexpr int kNoId = 0x7fffffff;  // "no candidate": after every real (v, id)
+constexpr int kCandCap = 64;        // per-warp candidate buffer (logits at or above the threshold)
 
 struct VI {
     float v;
@@ -55,8 +61,22 @@ __device__ __forceinline__ MS ms_merge(MS a, MS b) {
     return MS{M, a.s * __expf(a.m - M) + b.s * __expf(b.m - M)};
 }
 
+// Descending bitonic sort of one float per lane across the warp.
+__device__ __forceinline__ float warp_sort_desc(float x, int lane) {
+#pragma unroll
+    for (int k = 2; k <= 32; k <<= 1) {
+#pragma unroll
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            const float y = __shfl_xor_sync(0xffffffffu, x, j);
+            const bool keep_max = ((lane & j) == 0) == ((lane & k) == 0);
+            x = keep_max ? fmaxf(x, y) : fminf(x, y);
+        }
+    }
+    return x;
+}
+
 template <bool kVec>
-__global__ void __launch_bounds__(kAccThreads)
+__global__ void __launch_bounds__(kAccThreads, 3)
 accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *__restrict__ cand,
             MS *__restrict__ part) {
     const long long blk = blockIdx.x;
@@ -65,14 +85,19 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
     const float *row = logits + r * (long long)V;
     const int c0 = chunk * kAccChunk;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    constexpr float kL2E = 1.4426950408889634f;
+
+    __shared__ MS sms[kAccThreads / 32];
+    __shared__ VI s_wtop[kAccThreads / 32][RS_MAX_BETA];  // each warp's best beta
+    __shared__ VI s_cbuf[kAccThreads / 32][kCandCap];     // each warp's candidates
+    __shared__ int s_cnt[kAccThreads / 32];
+    if (lane == 0) s_cnt[warp] = 0;
 
     float v[kAccVpt];
-    int base[kAccVpt / 4];  // first id of each float4 group (ids are base + 0..3)
     if (kVec) {
 #pragma unroll
         for (int j = 0; j < kAccVpt / 4; ++j) {
-            int idx = c0 + (j * kAccThreads + tid) * 4;
-            base[j] = idx;
+            const int idx = c0 + (j * kAccThreads + tid) * 4;
             float4 x;
             if (idx + 3 < V) {
                 x = ldg_stream4(reinterpret_cast<const float4 *>(row + idx));
@@ -90,28 +115,29 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
     } else {
 #pragma unroll
         for (int j = 0; j < kAccVpt; ++j) {
-            int idx = c0 + j * kAccThreads + tid;
+            const int idx = c0 + j * kAccThreads + tid;
             v[j] = idx < V ? ldg_stream(row + idx) : -INFINITY;
         }
     }
+    // logit id of register j (padding slots have ids >= V)
     auto id_of = [&](int j) -> int {
-        if (kVec) return base[j >> 2] + (j & 3);
+        if (kVec) return c0 + ((j >> 2) * kAccThreads + tid) * 4 + (j & 3);
         return c0 + j * kAccThreads + tid;
     };
-    // padded slots (id >= V) are never candidates
-    auto valid = [&](int j) -> bool { return id_of(j) < V; };
 
-    __shared__ VI sw[kAccThreads / 32];
-    __shared__ MS sms[kAccThreads / 32];
-
-    // (max, sum) for the row's log-sum-exp
-    float mx = -INFINITY;
+    // lane maximum (pairwise) and (max, sum e^(z - max)) for the log-sum-exp
+    float m8[8];
 #pragma unroll
-    for (int j = 0; j < kAccVpt; ++j) mx = fmaxf(mx, v[j]);
+    for (int q = 0; q < 8; ++q) m8[q] = fmaxf(fmaxf(v[q], v[q + 8]), fmaxf(v[q + 16], v[q + 24]));
+    const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                           fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
     MS t{mx, 0.f};
     if (mx != -INFINITY) {
+        const float nb = -mx * kL2E;
+        float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int j = 0; j < kAccVpt; ++j) t.s += __expf(v[j] - mx);
+        for (int j = 0; j < kAccVpt; ++j) s4[j & 3] += sm100::ex2(fmaf(v[j], kL2E, nb));
+        t.s = (s4[0] + s4[1]) + (s4[2] + s4[3]);
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -120,29 +146,74 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
     }
     if (lane == 0) sms[warp] = t;
 
-    // beta rounds: best (v, id) strictly after the previous round's winner
-    VI prev{INFINITY, -1};
-    for (int k = 0; k < beta; ++k) {
-        VI best{-INFINITY, kNoId};
+    // ---- the warp's best beta, exactly, in (logit desc, id asc) order ----
+    // The beta-th largest lane maximum is a lower bound on the warp's beta-th
+    // largest logit (the beta lanes it ranks each hold a logit >= it), so
+    // only logits >= it can be in the warp's best beta.  Those few are
+    // appended to a shared buffer and ranked; if ties overflow the buffer,
+    // every logit of the warp is ranked instead.
+    const float thr = __shfl_sync(0xffffffffu, warp_sort_desc(mx, lane), beta - 1);
+    __syncwarp();
 #pragma unroll
-        for (int j = 0; j < kAccVpt; ++j) {
-            int id = id_of(j);
-            if (valid(j) && vi_before(prev.v, prev.i, v[j], id) && vi_before(v[j], id, best.v, best.i))
-                best = VI{v[j], id};
+    for (int j = 0; j < kAccVpt; ++j) {
+        if (v[j] >= thr) {
+            const int id = id_of(j);
+            if (id < V) {
+                const int p = atomicAdd(&s_cnt[warp], 1);
+                if (p < kCandCap) s_cbuf[warp][p] = VI{v[j], id};
+            }
         }
-        best = warp_vi_best(best);
-        __syncthreads();  // previous round's readers of sw are done
-        if (lane == 0) sw[warp] = best;
-        __syncthreads();
-        VI w = lane < kAccThreads / 32 ? sw[lane] : VI{-INFINITY, kNoId};
-        w = warp_vi_best(w);
-        prev = w;  // identical in every warp
-        if (tid == 0) cand[blk * beta + k] = w;
     }
-    if (tid == 0) {
-        MS a = sms[0];
-        for (int w = 1; w < kAccThreads / 32; ++w) a = ms_merge(a, sms[w]);
-        part[blk] = a;
+    __syncwarp();
+    const int total = s_cnt[warp];
+    VI prev{INFINITY, -1};
+    if (total <= kCandCap) {
+        for (int k = 0; k < beta; ++k) {
+            VI best{-INFINITY, kNoId};
+            for (int q = lane; q < total; q += 32) {
+                const VI x = s_cbuf[warp][q];
+                if (vi_before(prev.v, prev.i, x.v, x.i) && vi_before(x.v, x.i, best.v, best.i)) best = x;
+            }
+            best = warp_vi_best(best);
+            prev = best;
+            if (lane == 0) s_wtop[warp][k] = best;
+        }
+    } else {
+        for (int k = 0; k < beta; ++k) {
+            VI best{-INFINITY, kNoId};
+#pragma unroll
+            for (int j = 0; j < kAccVpt; ++j) {
+                const int id = id_of(j);
+                if (id < V && vi_before(prev.v, prev.i, v[j], id) && vi_before(v[j], id, best.v, best.i))
+                    best = VI{v[j], id};
+            }
+            best = warp_vi_best(best);
+            prev = best;
+            if (lane == 0) s_wtop[warp][k] = best;
+        }
+    }
+    __syncthreads();
+
+    // ---- warp 0 merges the warps' lists into the chunk's best beta ----
+    if (warp == 0) {
+        constexpr int kW = kAccThreads / 32;
+        VI prevb{INFINITY, -1};
+        for (int k = 0; k < beta; ++k) {
+            VI best{-INFINITY, kNoId};
+            for (int q = lane; q < kW * beta; q += 32) {
+                const VI x = s_wtop[q / beta][q % beta];
+                if (x.i != kNoId && vi_before(prevb.v, prevb.i, x.v, x.i) && vi_before(x.v, x.i, best.v, best.i))
+                    best = x;
+            }
+            best = warp_vi_best(best);
+            prevb = best;
+            if (lane == 0) cand[blk * beta + k] = best;
+        }
+        if (lane == 0) {
+            MS a = sms[0];
+            for (int w = 1; w < kW; ++w) a = ms_merge(a, sms[w]);
+            part[blk] = a;
+        }
     }
 }
 

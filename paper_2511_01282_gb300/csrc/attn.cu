@@ -81,9 +81,20 @@ attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_
 }
 
 // Block c merges the split segment whose first piece is c's last piece.
-__global__ void __launch_bounds__(256)
+// Phase 1: one thread per row forms M = max_p m_p and the weights
+// e^(m_p - M) / sum_p e^(m_p - M) l_p in shared memory.  Phase 2: the block
+// sweeps (row, 4 head-dim columns) items with float4 loads of the partial O.
+constexpr int kCombThreads = 256;
+constexpr int kMaxPieces = 1024;
+constexpr int kFastPieces = 16;  // pieces whose weights fit the shared table
+
+__global__ void __launch_bounds__(kCombThreads)
 attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
     extern __shared__ int s_pref[];
+    __shared__ int s_slot[kMaxPieces];
+    __shared__ float s_w[kFastPieces][kBM];
+    __shared__ float s_M[kBM], s_L[kBM];
+    __shared__ int s_np;
     unit_prefix(info, a.B, s_pref);
     const long long W = s_pref[a.B];
     const long long Gc = gridDim.x, c = blockIdx.x;
@@ -97,38 +108,68 @@ attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
     const long long seg_end = seg_start + ri.nt;
     if (!(seg_start >= u0 && seg_end > u1)) return;  // not the first owner of a split segment
     const long long c1 = owner_of(seg_end - 1, W, Gc);
-
+    if (threadIdx.x == 0) {
+        int np = 0;
+        for (long long cc = c; cc <= c1 && np < kMaxPieces; ++cc) {
+            const long long lo = range_lo(cc, W, Gc);
+            if (lo == range_lo(cc + 1, W, Gc)) continue;  // empty range: no piece
+            s_slot[np++] = (int)(2 * cc + (seg_start > lo ? 1 : 0));
+        }
+        s_np = np;
+    }
+    __syncthreads();
+    const int np = s_np;
     const int G = a.Hq / a.Hkv;
     const int n0 = a.node_off[b];
     const int N = a.node_off[b + 1] - n0;
     const int kvh = seg / ri.mt, mtile = seg - kvh * ri.mt;
     const int rows = min(kBM, N * G - mtile * kBM);
     const int D = a.D;
-    for (int x = threadIdx.x; x < rows * D; x += blockDim.x) {
-        const int r = x / D, d = x - r * D;
+    const bool fast = np <= kFastPieces;
+    // phase 1: per-row maximum, normaliser and (fast path) weights
+    for (int r = threadIdx.x; r < rows; r += kCombThreads) {
         float M = -INFINITY;
-        for (long long cc = c; cc <= c1; ++cc) {
-            const long long lo = range_lo(cc, W, Gc);
-            if (lo == range_lo(cc + 1, W, Gc)) continue;
-            const int slot = (int)(2 * cc + (seg_start > lo ? 1 : 0));
-            M = fmaxf(M, a.part_m[(long long)slot * kBM + r]);
+        for (int p = 0; p < np; ++p) M = fmaxf(M, a.part_m[(long long)s_slot[p] * kBM + r]);
+        float L = 0.f;
+        for (int p = 0; p < np; ++p) {
+            const long long prow = (long long)s_slot[p] * kBM + r;
+            const float m = a.part_m[prow];
+            const float w = m == -INFINITY ? 0.f : __expf(m - M);
+            L += w * a.part_l[prow];
+            if (fast) s_w[p][r] = w;
         }
-        float L = 0.f, O = 0.f;
-        for (long long cc = c; cc <= c1; ++cc) {
-            const long long lo = range_lo(cc, W, Gc);
-            if (lo == range_lo(cc + 1, W, Gc)) continue;
-            const int slot = (int)(2 * cc + (seg_start > lo ? 1 : 0));
-            const float m = a.part_m[(long long)slot * kBM + r];
-            if (m == -INFINITY) continue;
-            const float w = __expf(m - M);
-            L += w * a.part_l[(long long)slot * kBM + r];
-            O += w * a.part_o[((long long)slot * kBM + r) * D + d];
+        s_M[r] = M;
+        s_L[r] = L;
+        if (fast)
+            for (int p = 0; p < np; ++p) s_w[p][r] /= L;
+    }
+    __syncthreads();
+    // phase 2: outputs, four columns per item
+    const int d4 = D / 4;
+    for (int x = threadIdx.x; x < rows * d4; x += kCombThreads) {
+        const int r = x / d4, q = x - r * d4;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int p = 0; p < np; ++p) {
+            const long long prow = (long long)s_slot[p] * kBM + r;
+            float w;
+            if (fast) {
+                w = s_w[p][r];
+            } else {
+                const float m = a.part_m[prow];
+                w = m == -INFINITY ? 0.f : __expf(m - s_M[r]) / s_L[r];
+            }
+            if (w == 0.f) continue;
+            const float4 o = *reinterpret_cast<const float4 *>(a.part_o + prow * D + q * 4);
+            acc.x += w * o.x;
+            acc.y += w * o.y;
+            acc.z += w * o.z;
+            acc.w += w * o.w;
         }
         const int rr = mtile * kBM + r;
-        const int i = rr / G, h = kvh * G + (rr - (rr / G) * G);
+        const int i = rr / G, h = kvh * G + (rr - i * G);
         const long long orow = (long long)(n0 + i) * a.Hq + h;
-        a.out[orow * D + d] = O / L;
-        if (d == 0) a.lse[orow] = M + __logf(L);
+        *reinterpret_cast<float4 *>(a.out + orow * D + q * 4) = acc;
+        if (q == 0) a.lse[orow] = s_M[r] + __logf(s_L[r]);
     }
 }
 
@@ -199,7 +240,7 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     }
     RS_CHECK_ARG(B <= kAttnMaxB, "rs_tree_verify_attn: B=%d above %d", B, kAttnMaxB);
     RS_CHECK_ARG(kv_rows < (1ll << 31) - kBN, "rs_tree_verify_attn: kv_rows above 2^31");
-    RS_CHECK_ARG(isfinite(scale), "rs_tree_verify_attn: scale must be finite");
+    RS_CHECK_ARG(isfinite(scale) && scale > 0.f, "rs_tree_verify_attn: scale must be finite and > 0");
     RS_CHECK_ARG(B == 0 || (kv_off && ctx_len && node_off && status), "rs_tree_verify_attn: null request pointer");
     RS_CHECK_ARG(R == 0 || (q && parents && out && lse), "rs_tree_verify_attn: null row pointer");
     RS_CHECK_ARG(kv_rows == 0 || (k && v), "rs_tree_verify_attn: null KV pointer");
@@ -267,7 +308,7 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     else
         attn_tc_kernel<64><<<Gc, kAttnThreads, smem, st>>>(a, info, tmk, tmv);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/main");
-    attn_combine<<<Gc, 256, (size_t)(B + 1) * sizeof(int), st>>>(a, info);
+    attn_combine<<<Gc, kCombThreads, (size_t)(B + 1) * sizeof(int), st>>>(a, info);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/combine");
     return RS_OK;
 }

@@ -3,18 +3,24 @@
 //
 // One CTA per SM walks its contiguous range of KV-tile units (see attn.cu).
 // Within a CTA, warps are specialised:
-//   warp 4 (1 thread)  TMA: K and V tiles of 128 keys x D into a 2-stage
+//   warp 8 (1 thread)  TMA: K and V tiles of 128 keys x D into a 3-stage
 //                      ring of 128-byte-swizzled shared-memory buffers;
-//   warp 5 (1 thread)  MMA: S = Q K^T into one of two TMEM buffers, then
+//   warp 9 (1 thread)  MMA: S = Q K^T into one of two TMEM buffers, then
 //                      O += P V with P read from TMEM (bf16, written over
 //                      S by the softmax warps) and V from shared memory;
-//   warps 0-3          one thread per row of the 128-row tile: load Q, mask
+//   warps 0-7          two softmax warpgroups over the same 128 rows (the
+//                      TMEM lane of a warp is fixed by warp % 4), each
+//                      taking 64 of a tile's 128 keys; they agree on the
+//                      row maxima through a named barrier.  Per row: Q into
+//                      TMEM, mask
 //                      (prefix always visible, tree slots by the ancestor
 //                      bit set, other requests' keys never), online softmax in
 //                      base 2 with lazy rescaling of O (only when the running
 //                      maximum grows by more than 2^8), write P, and the
 //                      epilogue (final O / l and log-sum-exp, or a partial).
-// TMEM columns: O [0, D), S/P buffer b at [128 + 128 b, 256 + 128 b).
+// TMEM columns: O [0, D), S/P buffer b at [128 + 128 b, 256 + 128 b), Q
+// (bf16, two per column) at [384, 384 + D/2).  The MMA reads Q and P as
+// tensor-memory A operands; only K and V go through shared memory.
 // Every mbarrier wait is bounded: on a time-out the CTA raises an abort flag,
 // every role leaves its loop, in-flight copies and MMAs are drained (again
 // bounded), TMEM is released and RS_ST_TIMEOUT is OR-ed into the status of
@@ -32,19 +38,22 @@ namespace rs {
 constexpr int kBM = 128;  // (node, q-head-in-group) rows per tile
 constexpr int kBN = 128;  // keys per KV tile (one work unit)
 constexpr int kAncWords = RS_MAX_NODES / 32;
-constexpr int kAttnThreads = 192;
-constexpr int kNS = 2;                             // K/V ring stages
-constexpr int kTileBytes = kBM * 128 * 2;          // one 128 x 128 bf16 tile
-constexpr int kSmemQ = 0;
-constexpr int kSmemK = kTileBytes;
+constexpr int kSoftThreads = 256;  // two softmax warpgroups (warps 0-7)
+constexpr int kTmaWarp = 8, kMmaWarp = 9;
+constexpr int kAttnThreads = 320;
+constexpr int kNS = 3;                             // K/V ring stages
+constexpr int kTileBytes = kBN * 128 * 2;          // one 128-key x 128-dim bf16 tile
+constexpr int kSmemK = 0;
 constexpr int kSmemV = kSmemK + kNS * kTileBytes;
 constexpr int kSmemBar = kSmemV + kNS * kTileBytes;
-constexpr int kNumBars = 3 * kNS + 8;
+constexpr int kNumBars = 3 * kNS + 12;
 constexpr int kSmemMisc = kSmemBar + kNumBars * 8;  // tmem base, abort flag
 constexpr int kSmemPref = kSmemMisc + 16;
-constexpr int kAttnMaxB = 8192;
+constexpr int kAttnMaxB = 4096;
 constexpr long long kWaitLimit = 4000000000ll;     // clock cycles (~2 s)
 constexpr uint32_t kTmemCols = 512;
+// TMEM columns: O [0, 128), S/P buffers [128, 256) and [256, 384), Q [384, 448)
+constexpr uint32_t kTmO = 0, kTmS = 128, kTmQ = 384;
 
 inline size_t attn_smem_bytes(int B) { return 1024 + kSmemPref + (size_t)(B + 1) * sizeof(int); }
 
@@ -172,6 +181,21 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t *>(&v);
 }
 
+// Warp-uniform bounded wait for the softmax warps: every lane waits, and the
+// warp gives up together if any lane gave up, so warp-wide instructions
+// (tcgen05.ld/st, vote) that follow always see the whole warp.
+__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
+    const bool ok = sm100::mbar_wait(bar, parity, abort, kWaitLimit);
+    return __all_sync(0xffffffffu, ok);
+}
+
+// The calling warp arrives once for all its 32 lanes (after every lane's
+// prior shared-memory and tensor-memory work is ordered by __syncwarp).
+__device__ __forceinline__ void warp_arrive(uint64_t *bar) {
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) sm100::mbar_arrive_cnt(bar, 32);
+}
+
 // ------------------------------------------------------------------ kernel
 template <int D>
 __global__ void __launch_bounds__(kAttnThreads, 1)
@@ -183,8 +207,9 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                                                             ~uintptr_t(1023));
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kSmemBar);
     uint64_t *kfull = bars, *vfull = bars + kNS, *kvempty = bars + 2 * kNS;
-    uint64_t *sfull = bars + 3 * kNS, *pfull = sfull + 2, *odone = pfull + 2, *qready = odone + 1;
+    uint64_t *sfull = bars + 3 * kNS, *pfull = sfull + 2, *odone = pfull + 2, *qready = odone + 2;
     uint64_t *ofree = qready + 1, *drain = ofree + 1;
+    uint64_t *mxready = drain + 1, *lready = mxready + 2;  // softmax warpgroup exchanges
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + kSmemMisc);
     volatile int *s_abort = reinterpret_cast<volatile int *>(smem + kSmemMisc + 4);
     int *s_pref = reinterpret_cast<int *>(smem + kSmemPref);
@@ -198,17 +223,21 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&sfull[s], 1);
-            mbar_init(&pfull[s], 128);
+            mbar_init(&pfull[s], kSoftThreads);
         }
-        mbar_init(odone, 1);
-        mbar_init(qready, 128);
-        mbar_init(ofree, 128);
+        mbar_init(&odone[0], 1);
+        mbar_init(&odone[1], 1);
+        mbar_init(qready, kSoftThreads);
+        mbar_init(ofree, kSoftThreads);
         mbar_init(drain, 1);
+        mbar_init(&mxready[0], kSoftThreads);
+        mbar_init(&mxready[1], kSoftThreads);
+        mbar_init(lready, kSoftThreads);
         *s_abort = 0;
         fence_mbar_init();
     }
-    if (warp == 5) tmem_alloc(s_tmem, kTmemCols);
-    if (warp == 4 && lane == 0) {
+    if (warp == kMmaWarp) tmem_alloc(s_tmem, kTmemCols);
+    if (warp == kTmaWarp && lane == 0) {
         prefetch_tmap(&tmk);
         prefetch_tmap(&tmv);
     }
@@ -222,7 +251,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
     constexpr uint32_t kTileTx = (uint32_t)kBN * D * 2;
     constexpr int kKB = D / 64;  // 64-column swizzle blocks per row
 
-    if (warp == 4) {
+    if (warp == kTmaWarp) {
         // ---------------------------------------------------------- TMA producer
         if (lane == 0) {
             long long g = 0;
@@ -255,12 +284,12 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                 }
             }
         }
-    } else if (warp == 5) {
+    } else if (warp == kMmaWarp) {
         // ---------------------------------------------------------- MMA issuer
         if (lane == 0) {
             constexpr uint32_t idS = idesc_bf16_f32(kBM, kBN, false);
             constexpr uint32_t idO = idesc_bf16_f32(kBM, D, true);
-            const uint32_t q_addr = smem_u32(smem + kSmemQ);
+            const uint32_t q_tm = tmem + kTmQ;
             long long g = 0;
             int piece = 0;
             bool ok = true;
@@ -269,12 +298,11 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                 if (!mbar_wait(&kfull[st], (uint32_t)((gt / kNS) & 1), s_abort, kWaitLimit)) return false;
                 tc_fence_after();
                 const uint32_t k_addr = smem_u32(smem + kSmemK + st * kTileBytes);
-                const uint32_t d_s = tmem + 128 + (uint32_t)(gt & 1) * 128;
+                const uint32_t d_s = tmem + kTmS + (uint32_t)(gt & 1) * 128;
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint32_t off = (uint32_t)((kk >> 2) * 16384 + (kk & 3) * 32);
-                    umma_ss(d_s, sdesc_sw128(q_addr + off, 16, 1024), sdesc_sw128(k_addr + off, 16, 1024), idS,
-                            kk > 0);
+                    umma_ts(d_s, q_tm + kk * 8, sdesc_sw128(k_addr + off, 16, 1024), idS, kk > 0);
                 }
                 umma_commit(&sfull[gt & 1]);
                 return true;
@@ -296,13 +324,13 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                         break;
                     tc_fence_after();
                     const uint32_t v_addr = smem_u32(smem + kSmemV + st * kTileBytes);
-                    const uint32_t p_tm = tmem + 128 + (uint32_t)(gt & 1) * 128;
+                    const uint32_t p_tm = tmem + kTmS + (uint32_t)(gt & 1) * 128;
 #pragma unroll
                     for (int ks = 0; ks < kBN / 16; ++ks)
-                        umma_ts(tmem, p_tm + ks * 8, sdesc_sw128(v_addr + ks * 2048, 16384, 1024), idO,
+                        umma_ts(tmem + kTmO, p_tm + ks * 8, sdesc_sw128(v_addr + ks * 2048, 16384, 1024), idO,
                                 (tl > 0 || ks > 0) ? 1u : 0u);
                     umma_commit(&kvempty[st]);
-                    umma_commit(odone);
+                    umma_commit(&odone[gt & 1]);
                 }
                 g += n;
                 u = pc.end;
@@ -315,12 +343,25 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
         }
     } else {
         // ---------------------------------------------------------- softmax / epilogue (rows)
-        const int r = tid;  // row of the tile == TMEM lane
-        const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
-        const float cexp = a.scale * 1.4426950408889634f;  // scores -> log2 domain
+        // PV of tile t commits odone[t & 1].  Once S of tile t has been seen
+        // complete, every PV up to t - 2 is complete (S_t is issued after
+        // PV_{t-2}), so odone[b] is at most one phase behind the tile this
+        // thread asks for: a parity wait is unambiguous even though the
+        // thread waits only when it must read O (a rescale or the epilogue).
+        // Warpgroup hw (0 or 1) owns keys [64 hw, 64 hw + 64) of every tile,
+        // O columns [hw D/2, (hw + 1) D/2) for rescales and the epilogue, and
+        // its own partial row sum; both keep the same reference maximum.
+        // The per-tile maxima and the final sums are exchanged through
+        // shared memory guarded by mbarriers (mxready[tile & 1], lready).
+        __shared__ float s_mx[2][2][kBM];  // [tile parity][warpgroup][row]
+        __shared__ float s_l[2][kBM];
+        const int r = tid & (kBM - 1);      // row of the tile == TMEM lane
+        const int hw = tid >> 7;            // warpgroup
+        const uint32_t lane_off = (uint32_t)((warp & 3) * 32) << 16;
+        const float cexp = a.scale * 1.4426950408889634f;  // scores -> log2 domain (scale > 0)
+        constexpr int kHalfO = D / 2;       // O columns per warpgroup
         long long g = 0;
         int piece = 0;
-        uint32_t odone_phase = 0;
         bool ok = true;
         for (long long u = u0; u < u1 && ok; ++piece) {
             const Piece pc = piece_at(info, s_pref, a.B, u, u0, u1, c);
@@ -332,21 +373,26 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
             const int i = valid ? rr / G : 0;
             const int h = pc.kvh * G + (valid ? rr - i * G : 0);
 
-            // Q row -> swizzled shared memory (rows past the tile's end are zero)
-            {
-                const uint4 *qp = reinterpret_cast<const uint4 *>(a.q + ((long long)(n0 + i) * a.Hq + h) * D);
+            // Q row -> TMEM (bf16 pairs, 64 elements per 32 columns; zero past the tile)
+            if (hw < D / 64) {
+                const uint4 *qp = reinterpret_cast<const uint4 *>(a.q + ((long long)(n0 + i) * a.Hq + h) * D) + hw * 8;
+                uint32_t x[32];
 #pragma unroll
-                for (int ch = 0; ch < D / 8; ++ch) {
-                    uint4 x = valid ? qp[ch] : make_uint4(0, 0, 0, 0);
-                    const int kb = ch >> 3, cc = ch & 7;
-                    *reinterpret_cast<uint4 *>(smem + kSmemQ + kb * 16384 + r * 128 + ((cc ^ (r & 7)) << 4)) = x;
+                for (int e = 0; e < 8; ++e) {
+                    const uint4 v = valid ? qp[e] : make_uint4(0, 0, 0, 0);
+                    x[4 * e + 0] = v.x;
+                    x[4 * e + 1] = v.y;
+                    x[4 * e + 2] = v.z;
+                    x[4 * e + 3] = v.w;
                 }
+                tmem_st32(tmem + lane_off + kTmQ + hw * 32, x);
+                tmem_wait_st();
             }
             uint32_t anc[kAncWords];
 #pragma unroll
             for (int w = 0; w < kAncWords; ++w) anc[w] = valid ? a.anc[(long long)(n0 + i) * kAncWords + w] : 0u;
-            fence_async_smem();
-            mbar_arrive(qready);
+            tc_fence_before();
+            warp_arrive(qready);
 
             float m_used = -INFINITY, l = 0.f;
             const int n = pc.j1 - pc.j0;
@@ -354,57 +400,60 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                 const long long gt = g + tl;
                 const int buf = (int)(gt & 1);
                 const int jt = pc.j0 + tl;
-                if (!(ok = mbar_wait(&sfull[buf], (uint32_t)((gt >> 1) & 1), s_abort, kWaitLimit))) break;
+                if (!(ok = warp_wait(&sfull[buf], (uint32_t)((gt >> 1) & 1), s_abort))) break;
                 tc_fence_after();
-                const uint32_t s_tm = tmem + lane_off + 128 + (uint32_t)buf * 128;
-                float s[kBN];
+                const uint32_t s_tm = tmem + lane_off + kTmS + (uint32_t)buf * 128;
+                float s[64];
 #pragma unroll
-                for (int ch = 0; ch < kBN / 32; ++ch) {
+                for (int ch = 0; ch < 2; ++ch) {
                     uint32_t x[32];
-                    tmem_ld32(s_tm + ch * 32, x);
+                    tmem_ld32(s_tm + hw * 64 + ch * 32, x);
                     tmem_wait_ld();
 #pragma unroll
                     for (int e = 0; e < 32; ++e) s[ch * 32 + e] = __uint_as_float(x[e]);
                 }
-                float mt = -INFINITY;
-                const int key0 = jt * kBN;
-                if (key0 + kBN <= S) {  // prefix-only tile: nothing to mask
+                // raw-score maximum over this half's visible keys
+                float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                const int key0 = jt * kBN + hw * 64;
+                if (key0 + 64 <= S) {  // prefix-only: nothing to mask
 #pragma unroll
-                    for (int j = 0; j < kBN; ++j) {
-                        s[j] *= cexp;
-                        mt = fmaxf(mt, s[j]);
-                    }
+                    for (int j = 0; j < 64; ++j) mx4[j & 3] = fmaxf(mx4[j & 3], s[j]);
                 } else {
 #pragma unroll
-                    for (int ch = 0; ch < kBN / 32; ++ch) {
+                    for (int ch = 0; ch < 2; ++ch) {
                         const uint32_t msk = tree_window(anc, key0 + ch * 32 - S);
 #pragma unroll
                         for (int e = 0; e < 32; ++e) {
-                            const float v = ((msk >> e) & 1u) ? s[ch * 32 + e] * cexp : -INFINITY;
+                            const float v = ((msk >> e) & 1u) ? s[ch * 32 + e] : -INFINITY;
                             s[ch * 32 + e] = v;
-                            mt = fmaxf(mt, v);
+                            mx4[e & 3] = fmaxf(mx4[e & 3], v);
                         }
                     }
                 }
-                if (tl > 0) {  // PV of the previous tile is complete: O may be rescaled
-                    if (!(ok = mbar_wait(odone, odone_phase & 1, s_abort, kWaitLimit))) break;
-                    ++odone_phase;
-                    tc_fence_after();
-                }
+                // exchange the two halves' maxima through an mbarrier (bounded
+                // wait: a named barrier could not give up if a peer aborted)
+                s_mx[buf][hw][r] = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+                warp_arrive(&mxready[buf]);
+                if (!(ok = warp_wait(&mxready[buf], (uint32_t)((gt >> 1) & 1), s_abort))) break;
+                const float mt = fmaxf(s_mx[buf][0][r], s_mx[buf][1][r]) * cexp;
                 // lazy rescale: move the reference maximum only when it grows by
                 // more than 2^8; tcgen05.ld/st are warp-wide, so the O pass runs
                 // when any row of the warp needs it (factor 1 for the others)
                 const bool grow = mt > m_used + 8.f;
                 const float corr = grow ? ex2(m_used - mt) : 1.f;  // 0 when m_used is -inf
                 if (tl > 0 && __any_sync(0xffffffffu, grow)) {
+                    const long long pv = gt - 1;  // O must hold PV of the previous tile
+                    if (!(ok = warp_wait(&odone[pv & 1], (uint32_t)((pv >> 1) & 1), s_abort))) break;
+                    tc_fence_after();
 #pragma unroll
-                    for (int ch = 0; ch < D / 32; ++ch) {
+                    for (int ch = 0; ch < kHalfO / 32; ++ch) {
                         uint32_t x[32];
-                        tmem_ld32(tmem + lane_off + ch * 32, x);
+                        const uint32_t o_tm = tmem + lane_off + kTmO + hw * kHalfO + ch * 32;
+                        tmem_ld32(o_tm, x);
                         tmem_wait_ld();
 #pragma unroll
                         for (int e = 0; e < 32; ++e) x[e] = __float_as_uint(__uint_as_float(x[e]) * corr);
-                        tmem_st32(tmem + lane_off + ch * 32, x);
+                        tmem_st32(o_tm, x);
                     }
                     tmem_wait_st();
                 }
@@ -412,65 +461,66 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                     l *= corr;
                     m_used = mt;
                 }
-                const float base = (m_used == -INFINITY) ? 0.f : m_used;
-                float sum = 0.f;
-                uint32_t pw[kBN / 2];
+                const float nb = (m_used == -INFINITY) ? 0.f : -m_used;
+                float sum4[4] = {0.f, 0.f, 0.f, 0.f};
+                uint32_t x[32];
 #pragma unroll
-                for (int j = 0; j < kBN / 2; ++j) {
-                    const float p0 = ex2(s[2 * j] - base), p1 = ex2(s[2 * j + 1] - base);
-                    sum += p0 + p1;
-                    pw[j] = pack_bf16x2(p0, p1);
+                for (int e = 0; e < 32; ++e) {
+                    const float p0 = ex2(fmaf(s[2 * e], cexp, nb));
+                    const float p1 = ex2(fmaf(s[2 * e + 1], cexp, nb));
+                    sum4[e & 3] += p0 + p1;
+                    x[e] = pack_bf16x2(p0, p1);
                 }
-                l += sum;
-#pragma unroll
-                for (int ch = 0; ch < kBN / 64; ++ch) {
-                    uint32_t x[32];
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) x[e] = pw[ch * 32 + e];
-                    tmem_st32(s_tm + ch * 32, x);
-                }
+                tmem_st32(s_tm + hw * 32, x);
+                l += (sum4[0] + sum4[1]) + (sum4[2] + sum4[3]);
                 tmem_wait_st();
                 tc_fence_before();
-                mbar_arrive(&pfull[buf]);
+                warp_arrive(&pfull[buf]);
             }
             if (!ok) break;
-            // epilogue: O of the last tile is complete
-            if (!(ok = mbar_wait(odone, odone_phase & 1, s_abort, kWaitLimit))) break;
-            ++odone_phase;
+            // epilogue: the row sum is the two warpgroups' partial sums
+            s_l[hw][r] = l;
+            warp_arrive(lready);
+            if (!(ok = warp_wait(lready, (uint32_t)(piece & 1), s_abort))) break;
+            const float lt = s_l[0][r] + s_l[1][r];
+            {
+                const long long pv = g + n - 1;  // wait for PV of the last tile
+                if (!(ok = warp_wait(&odone[pv & 1], (uint32_t)((pv >> 1) & 1), s_abort))) break;
+            }
             tc_fence_after();
             const long long orow = (long long)(n0 + i) * a.Hq + h;
             const long long prow = (long long)pc.slot * kBM + r;
-            const float inv = (l > 0.f) ? 1.f / l : 0.f;
+            const float f = pc.final ? ((lt > 0.f) ? 1.f / lt : 0.f) : 1.f;
 #pragma unroll
-            for (int ch = 0; ch < D / 32; ++ch) {
+            for (int ch = 0; ch < kHalfO / 32; ++ch) {
                 uint32_t x[32];
-                tmem_ld32(tmem + lane_off + ch * 32, x);
+                const int col = hw * kHalfO + ch * 32;
+                tmem_ld32(tmem + lane_off + kTmO + col, x);
                 tmem_wait_ld();
                 if (valid) {
-                    float4 *dst = pc.final ? reinterpret_cast<float4 *>(a.out + orow * D + ch * 32)
-                                           : reinterpret_cast<float4 *>(a.part_o + prow * D + ch * 32);
-                    const float f = pc.final ? inv : 1.f;
+                    float4 *dst = pc.final ? reinterpret_cast<float4 *>(a.out + orow * D + col)
+                                           : reinterpret_cast<float4 *>(a.part_o + prow * D + col);
 #pragma unroll
                     for (int e = 0; e < 8; ++e)
                         dst[e] = make_float4(__uint_as_float(x[4 * e]) * f, __uint_as_float(x[4 * e + 1]) * f,
                                              __uint_as_float(x[4 * e + 2]) * f, __uint_as_float(x[4 * e + 3]) * f);
                 }
             }
-            if (valid) {
+            if (valid && hw == 0) {
                 const float m_nat = m_used * 0.6931471805599453f;
                 if (pc.final) {
-                    a.lse[orow] = m_nat + __logf(l);
+                    a.lse[orow] = m_nat + __logf(lt);
                 } else {
                     a.part_m[prow] = m_used == -INFINITY ? -INFINITY : m_nat;
-                    a.part_l[prow] = l;
+                    a.part_l[prow] = lt;
                 }
             }
             tc_fence_before();
-            mbar_arrive(ofree);
+            warp_arrive(ofree);
             g += n;
             u = pc.end;
         }
-        if (!ok && r == 0) {
+        if (!ok && tid == 0) {
             for (long long u = u0; u < u1;) {  // flag every request this CTA touches
                 const Piece pc = piece_at(info, s_pref, a.B, u, u0, u1, c);
                 atomicOr(&a.status[pc.b], RS_ST_TIMEOUT);
@@ -479,7 +529,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
         }
     }
     __syncthreads();
-    if (warp == 5) {
+    if (warp == kMmaWarp) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
     }
