@@ -126,6 +126,17 @@ rs_status rs_entropy_gate(const float *logits, int R, int V, const int32_t *row_
                           int32_t *k_star, float *h_best, uint8_t *entropy_ok,
                           void *workspace, size_t workspace_bytes, void *stream);
 
+/* ================================================ rs_entropy_gate_rows ====
+ * The trigger of rs_entropy_gate (history push, H_k, C_k, k*, step 4) from
+ * row entropies computed elsewhere -- rs_accept's `entropy` output over the
+ * same logits -- instead of from the logits.  Arguments as rs_entropy_gate;
+ * `entropy` is an input here.  One kernel, no workspace.
+ */
+rs_status rs_entropy_gate_rows(const float *entropy, const int32_t *row_off,
+                               const uint8_t *row_commit, int B, rs_params p,
+                               float *hist, int32_t *hist_n, int32_t *k_star,
+                               float *h_best, uint8_t *entropy_ok, void *stream);
+
 /* ============================================= rs_entropy_gate_noalloc ====
  * Not from the paper (it has no counterpart): rs_entropy_gate for callers
  * that cannot allocate device memory -- for example code embedded in a
@@ -243,7 +254,12 @@ rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, const uint16
  *   topk   [R, beta]  ids in (logit desc, id asc) order;
  *   lse    [R] fp32   log-sum-exp of the row;
  *   p_tok  [R] fp32   probability of node r's token under its parent's row
- *                     (1 for the root, 0 in a malformed request).
+ *                     (1 for the root, 0 in a malformed request);
+ *   entropy [R] fp32 or NULL: when given, the row entropy in nats (Eq. 1,
+ *                     as rs_entropy_gate computes it) from the same pass over
+ *                     the logits.  The verify step's logits are the next
+ *                     step's trigger input, so passing this to
+ *                     rs_entropy_gate_rows saves the gate's own logits pass.
  * Decision outputs, per request b:
  *   acc_len [B]            accepted draft tokens on the winning path;
  *   acc_nodes [B, acc_cap] their local node indices in depth order, -1 padded;
@@ -266,9 +282,9 @@ rs_status rs_accept(const float *logits, int R, int V, const int32_t *node_off, 
                     const int32_t *tokens, const int32_t *parents, const uint8_t *source,
                     const int8_t *chain, const int32_t *sel_pos, const int64_t *tok_off,
                     rs_params p, int acc_cap, int32_t *argmax, int32_t *topk, float *lse,
-                    float *p_tok, int32_t *acc_len, int32_t *acc_nodes, int32_t *bonus,
-                    int32_t *winner, uint8_t *commit, float *scores, int32_t *status,
-                    void *workspace, size_t workspace_bytes, void *stream);
+                    float *p_tok, float *entropy, int32_t *acc_len, int32_t *acc_nodes,
+                    int32_t *bonus, int32_t *winner, uint8_t *commit, float *scores,
+                    int32_t *status, void *workspace, size_t workspace_bytes, void *stream);
 
 #ifdef __cplusplus
 }

@@ -2,21 +2,28 @@
 // and the look-ahead tolerance procedure), longest accepted path and winner
 // (Algorithm 1 l.13), EMA feedback (Eq. 4-5, Algorithm 1 l.15-22).
 //
-// Kernel 1 (accept_rows): one CTA per (row, 8192-logit chunk).  Each thread
-// holds 32 logits in registers; the CTA produces the chunk's (max, sum e^(z -
-// max)) pair and its beta best (logit, id) pairs in the total order (logit
-// desc, id asc).  Each warp first bounds its beta-th largest logit from below
-// by the beta-th largest of its 32 lane maxima (a warp bitonic sort), appends
-// the few logits at or above that bound to shared memory and ranks only those
+// Kernel 1 (accept_rows): three persistent CTAs per SM walk the (row,
+// 8192-logit chunk) work items; each thread copies the next item's 32
+// logits into a second shared-memory stage (cp.async) while it works on the
+// current item from registers.  Per item the CTA produces the chunk's (max,
+// sum e^(z - max)[, sum e^(z - max) (z - max)]) triple and its beta best
+// (logit, id) pairs in the total order (logit desc, id asc).  The beta-th largest of a warp's 32 lane maxima (warp
+// bitonic sort) bounds the chunk's beta-th largest logit from below, and so
+// does the largest such bound over the warps; the few logits at or above it
+// are appended to shared memory and one warp (rotating over items) ranks them
 // by beta rounds of a "best after the previous winner" warp reduction (exact;
-// with many ties at the bound it ranks all of the warp's logits instead);
-// warp 0 merges the eight lists.  No dynamic register indexing.
-// Kernel 2 (accept_decide): one CTA per request.  Warps merge the chunk
-// candidates of each row (argmax, top-beta, lse); then the block checks the
-// tree, verifies model nodes (each thread walks its own root path), runs the
-// look-ahead procedure per chain (one thread per chain), picks the winner and
-// updates the scores.
+// with many ties at the bound every warp ranks its own logits and that warp
+// merges the lists).
+// No dynamic register indexing.
+// Kernel 2 (accept_merge): one warp per row merges the chunk results into
+// argmax, top-beta, log-sum-exp and (optionally) the row entropy.
+// Kernel 3 (accept_decide): one CTA per request checks the tree, verifies
+// model nodes (each thread walks its own root path), runs the look-ahead
+// procedure per chain (one thread per chain), picks the winner and updates
+// the scores.
 #include <math.h>
+
+#include <algorithm>
 
 #include "common.cuh"
 #include "sm100.cuh"
@@ -50,15 +57,23 @@ __device__ __forceinline__ VI warp_vi_best(VI a) {
     return a;
 }
 
+// (max m, sum e^(z-m), sum e^(z-m) (z-m)) of a set of logits: the row's
+// log-sum-exp is m + ln s and its entropy ln s - w / s.
 struct MS {
-    float m, s;
+    float m, s, w;
 };
 
 __device__ __forceinline__ MS ms_merge(MS a, MS b) {
     if (a.s == 0.f) return b;
     if (b.s == 0.f) return a;
-    float M = fmaxf(a.m, b.m);
-    return MS{M, a.s * __expf(a.m - M) + b.s * __expf(b.m - M)};
+    const float M = fmaxf(a.m, b.m);
+    const float ca = __expf(a.m - M), cb = __expf(b.m - M);
+    return MS{M, a.s * ca + b.s * cb, ca * (a.w + a.s * (a.m - M)) + cb * (b.w + b.s * (b.m - M))};
+}
+
+__device__ __forceinline__ MS ms_shfl(MS a, int o) {
+    return MS{__shfl_xor_sync(0xffffffffu, a.m, o), __shfl_xor_sync(0xffffffffu, a.s, o),
+              __shfl_xor_sync(0xffffffffu, a.w, o)};
 }
 
 // Descending bitonic sort of one float per lane across the warp.
@@ -75,38 +90,51 @@ __device__ __forceinline__ float warp_sort_desc(float x, int lane) {
     return x;
 }
 
+// cp.async: per-thread asynchronous global -> shared copies.  A thread's
+// wait_group only waits for its own copies, so no wait depends on another
+// thread.
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(sm100::smem_u32(smem)), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async4(void *smem, const void *gmem) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(sm100::smem_u32(smem)), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+
+// Start copying the logits this thread will hold of work item `item` = (row,
+// chunk) into `stage` (the same slots it later reads; ids >= V are skipped).
 template <bool kVec>
-__global__ void __launch_bounds__(kAccThreads, 3)
-accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *__restrict__ cand,
-            MS *__restrict__ part) {
-    const long long blk = blockIdx.x;
-    const long long r = blk / nchunks;
-    const int chunk = (int)(blk - r * nchunks);
+__device__ __forceinline__ void fetch_item(const float *__restrict__ logits, int V, int nchunks, long long item,
+                                           float *stage) {
+    const long long r = item / nchunks;
+    const int c0 = (int)(item - r * nchunks) * kAccChunk;
     const float *row = logits + r * (long long)V;
-    const int c0 = chunk * kAccChunk;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    constexpr float kL2E = 1.4426950408889634f;
-
-    __shared__ MS sms[kAccThreads / 32];
-    __shared__ VI s_wtop[kAccThreads / 32][RS_MAX_BETA];  // each warp's best beta
-    __shared__ VI s_cbuf[kAccThreads / 32][kCandCap];     // each warp's candidates
-    __shared__ int s_cnt[kAccThreads / 32];
-    if (lane == 0) s_cnt[warp] = 0;
-
-    float v[kAccVpt];
+    const int tid = threadIdx.x;
     if (kVec) {
 #pragma unroll
         for (int j = 0; j < kAccVpt / 4; ++j) {
-            const int idx = c0 + (j * kAccThreads + tid) * 4;
-            float4 x;
-            if (idx + 3 < V) {
-                x = ldg_stream4(reinterpret_cast<const float4 *>(row + idx));
-            } else {
-                x.x = idx + 0 < V ? row[idx + 0] : -INFINITY;
-                x.y = idx + 1 < V ? row[idx + 1] : -INFINITY;
-                x.z = idx + 2 < V ? row[idx + 2] : -INFINITY;
-                x.w = -INFINITY;
-            }
+            const int off = (j * kAccThreads + tid) * 4;
+            if (c0 + off < V) cp_async16(stage + off, row + c0 + off);  // V % 4 == 0: whole float4
+        }
+    } else {
+#pragma unroll
+        for (int j = 0; j < kAccVpt; ++j) {
+            const int off = j * kAccThreads + tid;
+            if (c0 + off < V) cp_async4(stage + off, row + c0 + off);
+        }
+    }
+}
+
+template <bool kVec>
+__device__ __forceinline__ void read_item(const float *stage, int V, int c0, float (&v)[kAccVpt]) {
+    const int tid = threadIdx.x;
+    if (kVec) {
+#pragma unroll
+        for (int j = 0; j < kAccVpt / 4; ++j) {
+            const int off = (j * kAccThreads + tid) * 4;
+            float4 x = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+            if (c0 + off < V) x = *reinterpret_cast<const float4 *>(stage + off);
             v[4 * j + 0] = x.x;
             v[4 * j + 1] = x.y;
             v[4 * j + 2] = x.z;
@@ -115,70 +143,126 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
     } else {
 #pragma unroll
         for (int j = 0; j < kAccVpt; ++j) {
-            const int idx = c0 + j * kAccThreads + tid;
-            v[j] = idx < V ? ldg_stream(row + idx) : -INFINITY;
+            const int off = j * kAccThreads + tid;
+            v[j] = c0 + off < V ? stage[off] : -INFINITY;
         }
     }
+}
+
+struct RowsShared {
+    MS sms[kAccThreads / 32];
+    float thr[kAccThreads / 32];
+    VI wtop[kAccThreads / 32][RS_MAX_BETA];  // per-warp lists (tie fallback)
+    VI cbuf[kCandCap];                       // the chunk's candidates
+    int cnt;
+};
+
+// One work item on the logits in registers: the chunk's (max, sum e, sum e
+// (z - max)) triple and its best beta candidates.
+// `rw` is the warp that ranks the candidates and writes the item's results
+// (rotated over items).  `sh` alternates between two copies over items, so no
+// barrier is needed at the end: a copy is next written two items later, after
+// every thread has passed the first barrier of the item in between.
+template <bool kVec, bool kEnt>
+__device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int nchunks, int beta, long long blk,
+                                          VI *__restrict__ cand, MS *__restrict__ part, RowsShared &sh, int rw) {
+    const int c0 = (int)(blk % nchunks) * kAccChunk;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    constexpr float kL2E = 1.4426950408889634f;
+    MS *sms = sh.sms;
+    float *s_thr = sh.thr;
+    auto &s_wtop = sh.wtop;
+    VI *s_cbuf = sh.cbuf;
+    int &s_cnt = sh.cnt;
+    if (tid == 0) s_cnt = 0;
+
     // logit id of register j (padding slots have ids >= V)
     auto id_of = [&](int j) -> int {
         if (kVec) return c0 + ((j >> 2) * kAccThreads + tid) * 4 + (j & 3);
         return c0 + j * kAccThreads + tid;
     };
 
-    // lane maximum (pairwise) and (max, sum e^(z - max)) for the log-sum-exp
+    // lane maximum (pairwise), then the warp maximum from the sorted lane
+    // maxima (the sort also gives the top-beta threshold below); every lane
+    // exponentiates against the warp maximum, so the warp's (max, sum e, sum
+    // e (z - max)) triple is a plain warp sum.
     float m8[8];
 #pragma unroll
     for (int q = 0; q < 8; ++q) m8[q] = fmaxf(fmaxf(v[q], v[q + 8]), fmaxf(v[q + 16], v[q + 24]));
     const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
                            fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
-    MS t{mx, 0.f};
-    if (mx != -INFINITY) {
-        const float nb = -mx * kL2E;
+    const float sorted = warp_sort_desc(mx, lane);
+    const float wmax = __shfl_sync(0xffffffffu, sorted, 0);
+    const float thr_w = __shfl_sync(0xffffffffu, sorted, beta - 1);
+    MS t{wmax, 0.f, 0.f};
+    if (wmax != -INFINITY) {
         float s4[4] = {0.f, 0.f, 0.f, 0.f};
+        float w4[4] = {0.f, 0.f, 0.f, 0.f};
+        if (kEnt) {  // also sum e (z - m) for the row entropy
 #pragma unroll
-        for (int j = 0; j < kAccVpt; ++j) s4[j & 3] += sm100::ex2(fmaf(v[j], kL2E, nb));
-        t.s = (s4[0] + s4[1]) + (s4[2] + s4[3]);
-    }
+            for (int j = 0; j < kAccVpt; ++j) {
+                const float d = fmaxf(v[j] - wmax, -1e30f);  // -inf -> -1e30: e = 0, e*d = 0
+                const float e = sm100::ex2(d * kL2E);
+                s4[j & 3] += e;
+                w4[j & 3] = fmaf(e, d, w4[j & 3]);
+            }
+        } else {
+            const float nb = -wmax * kL2E;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        MS u{__shfl_xor_sync(0xffffffffu, t.m, o), __shfl_xor_sync(0xffffffffu, t.s, o)};
-        t = ms_merge(t, u);
+            for (int j = 0; j < kAccVpt; ++j) s4[j & 3] += sm100::ex2(fmaf(v[j], kL2E, nb));
+        }
+        float ss = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+        float ww = (w4[0] + w4[1]) + (w4[2] + w4[3]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            ss += __shfl_xor_sync(0xffffffffu, ss, o);
+            if (kEnt) ww += __shfl_xor_sync(0xffffffffu, ww, o);
+        }
+        t.s = ss;
+        t.w = ww;
     }
     if (lane == 0) sms[warp] = t;
 
-    // ---- the warp's best beta, exactly, in (logit desc, id asc) order ----
-    // The beta-th largest lane maximum is a lower bound on the warp's beta-th
-    // largest logit (the beta lanes it ranks each hold a logit >= it), so
-    // only logits >= it can be in the warp's best beta.  Those few are
-    // appended to a shared buffer and ranked; if ties overflow the buffer,
-    // every logit of the warp is ranked instead.
-    const float thr = __shfl_sync(0xffffffffu, warp_sort_desc(mx, lane), beta - 1);
-    __syncwarp();
+    // ---- the chunk's best beta, exactly, in (logit desc, id asc) order ----
+    // A warp's beta-th largest lane maximum T_w is a lower bound on that
+    // warp's beta-th largest logit, hence on the chunk's beta-th largest
+    // logit; so is T = max_w T_w.  Only logits >= T can be in the chunk's
+    // best beta: they are appended to one shared buffer and ranked by warp 0.
+    // If ties overflow the buffer, every warp ranks its own logits and warp 0
+    // merges the eight lists instead.
+    if (lane == 0) s_thr[warp] = thr_w;
+    __syncthreads();
+    float thr = s_thr[0];
+#pragma unroll
+    for (int w = 1; w < kAccThreads / 32; ++w) thr = fmaxf(thr, s_thr[w]);
 #pragma unroll
     for (int j = 0; j < kAccVpt; ++j) {
         if (v[j] >= thr) {
             const int id = id_of(j);
             if (id < V) {
-                const int p = atomicAdd(&s_cnt[warp], 1);
-                if (p < kCandCap) s_cbuf[warp][p] = VI{v[j], id};
+                const int p = atomicAdd(&s_cnt, 1);
+                if (p < kCandCap) s_cbuf[p] = VI{v[j], id};
             }
         }
     }
-    __syncwarp();
-    const int total = s_cnt[warp];
-    VI prev{INFINITY, -1};
+    __syncthreads();
+    const int total = s_cnt;
     if (total <= kCandCap) {
-        for (int k = 0; k < beta; ++k) {
-            VI best{-INFINITY, kNoId};
-            for (int q = lane; q < total; q += 32) {
-                const VI x = s_cbuf[warp][q];
-                if (vi_before(prev.v, prev.i, x.v, x.i) && vi_before(x.v, x.i, best.v, best.i)) best = x;
+        if (warp == rw) {
+            VI prev{INFINITY, -1};
+            for (int k = 0; k < beta; ++k) {
+                VI best{-INFINITY, kNoId};
+                for (int q = lane; q < total; q += 32) {
+                    const VI x = s_cbuf[q];
+                    if (vi_before(prev.v, prev.i, x.v, x.i) && vi_before(x.v, x.i, best.v, best.i)) best = x;
+                }
+                best = warp_vi_best(best);
+                prev = best;
+                if (lane == 0) cand[blk * beta + k] = best;
             }
-            best = warp_vi_best(best);
-            prev = best;
-            if (lane == 0) s_wtop[warp][k] = best;
         }
     } else {
+        VI prev{INFINITY, -1};
         for (int k = 0; k < beta; ++k) {
             VI best{-INFINITY, kNoId};
 #pragma unroll
@@ -191,44 +275,115 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
             prev = best;
             if (lane == 0) s_wtop[warp][k] = best;
         }
-    }
-    __syncthreads();
-
-    // ---- warp 0 merges the warps' lists into the chunk's best beta ----
-    if (warp == 0) {
-        constexpr int kW = kAccThreads / 32;
-        VI prevb{INFINITY, -1};
-        for (int k = 0; k < beta; ++k) {
-            VI best{-INFINITY, kNoId};
-            for (int q = lane; q < kW * beta; q += 32) {
-                const VI x = s_wtop[q / beta][q % beta];
-                if (x.i != kNoId && vi_before(prevb.v, prevb.i, x.v, x.i) && vi_before(x.v, x.i, best.v, best.i))
-                    best = x;
+        __syncthreads();
+        if (warp == rw) {
+            constexpr int kW = kAccThreads / 32;
+            VI prevb{INFINITY, -1};
+            for (int k = 0; k < beta; ++k) {
+                VI best{-INFINITY, kNoId};
+                for (int q = lane; q < kW * beta; q += 32) {
+                    const VI x = s_wtop[q / beta][q % beta];
+                    if (x.i != kNoId && vi_before(prevb.v, prevb.i, x.v, x.i) &&
+                        vi_before(x.v, x.i, best.v, best.i))
+                        best = x;
+                }
+                best = warp_vi_best(best);
+                prevb = best;
+                if (lane == 0) cand[blk * beta + k] = best;
             }
-            best = warp_vi_best(best);
-            prevb = best;
-            if (lane == 0) cand[blk * beta + k] = best;
         }
+    }
+    if (warp == rw && lane == 0) {
+        MS a = sms[0];
+        for (int w = 1; w < kAccThreads / 32; ++w) a = ms_merge(a, sms[w]);
+        part[blk] = a;
+    }
+}
+
+// Persistent over work items: while a CTA works on item i, the copies of
+// item i + gridDim.x into the other shared-memory stage are in flight.
+constexpr int kRowsStages = 2;
+constexpr size_t kRowsSmem = (size_t)kRowsStages * kAccChunk * sizeof(float);
+
+template <bool kVec, bool kEnt>
+__global__ void __launch_bounds__(kAccThreads, 3)
+accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, long long n_items,
+            VI *__restrict__ cand, MS *__restrict__ part) {
+    __shared__ RowsShared sh[2];
+    extern __shared__ __align__(16) float s_stage[];  // kRowsStages x kAccChunk
+    const long long step = gridDim.x;
+    long long item = blockIdx.x;
+    if (item < n_items) fetch_item<kVec>(logits, V, nchunks, item, s_stage);
+    cp_async_commit();
+    for (int k = 0; item < n_items; ++k, item += step) {
+        float *cur = s_stage + (k & 1) * kAccChunk;
+        float *nxt = s_stage + ((k + 1) & 1) * kAccChunk;
+        if (item + step < n_items) fetch_item<kVec>(logits, V, nchunks, item + step, nxt);
+        cp_async_commit();
+        cp_async_wait_1();  // this thread's copies of `item` have landed
+        float v[kAccVpt];
+        read_item<kVec>(cur, V, (int)(item % nchunks) * kAccChunk, v);
+        rows_item<kVec, kEnt>(v, V, nchunks, beta, item, cand, part, sh[k & 1], k % (kAccThreads / 32));
+    }
+}
+
+// Row statistics: one warp per row merges the chunk candidates (loaded
+// once into registers, <= 32 * kCandPerLane) by beta rounds of a warp-wide
+// "best after the previous winner" reduction, and the chunk (m, s, w)
+// triples into the log-sum-exp (and the entropy when asked).
+constexpr int kMergeThreads = 256;
+constexpr int kCandPerLane = 8;
+
+__global__ void __launch_bounds__(kMergeThreads)
+accept_merge(const VI *__restrict__ cand, const MS *__restrict__ part, int nchunks, int beta, int R,
+             int32_t *__restrict__ argmax, int32_t *__restrict__ topk, float *__restrict__ lse,
+             float *__restrict__ entropy) {
+    const int lane = threadIdx.x & 31;
+    const long long r = (long long)blockIdx.x * (kMergeThreads / 32) + (threadIdx.x >> 5);
+    if (r >= R) return;
+    MS ms{-INFINITY, 0.f, 0.f};
+    for (int c = lane; c < nchunks; c += 32) ms = ms_merge(ms, part[r * nchunks + c]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) ms = ms_merge(ms, ms_shfl(ms, o));
+    const int ncand = nchunks * beta;
+    VI cv[kCandPerLane];
+#pragma unroll
+    for (int q = 0; q < kCandPerLane; ++q) {
+        const int c = lane + 32 * q;
+        cv[q] = c < ncand ? cand[r * ncand + c] : VI{-INFINITY, kNoId};
+    }
+    VI prev{INFINITY, -1};
+    for (int k = 0; k < beta; ++k) {
+        VI best{-INFINITY, kNoId};
+#pragma unroll
+        for (int q = 0; q < kCandPerLane; ++q) {
+            const VI x = cv[q];
+            if (x.i != kNoId && vi_before(prev.v, prev.i, x.v, x.i) && vi_before(x.v, x.i, best.v, best.i))
+                best = x;
+        }
+        best = warp_vi_best(best);
+        prev = best;
         if (lane == 0) {
-            MS a = sms[0];
-            for (int w = 1; w < kW; ++w) a = ms_merge(a, sms[w]);
-            part[blk] = a;
+            const int id = best.i == kNoId ? -1 : best.i;
+            topk[r * beta + k] = id;
+            if (k == 0) argmax[r] = id;
         }
+    }
+    if (lane == 0) {
+        lse[r] = ms.s > 0.f ? ms.m + __logf(ms.s) : -INFINITY;
+        if (entropy) entropy[r] = ms.s > 0.f ? (__logf(ms.s) - ms.w / ms.s) : 0.f;
     }
 }
 
 constexpr int kDecThreads = 512;
-// candidates per lane when a warp merges one row: nchunks * beta <= 32 * 8
-constexpr int kCandPerLane = 8;
 
 __global__ void __launch_bounds__(kDecThreads)
-accept_decide(const float *__restrict__ logits, int V, int nchunks, const VI *__restrict__ cand,
-              const MS *__restrict__ part, const int32_t *__restrict__ node_off,
+accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict__ node_off,
               const int32_t *__restrict__ tokens, const int32_t *__restrict__ parents,
               const uint8_t *__restrict__ source, const int8_t *__restrict__ chain,
               const int32_t *__restrict__ sel_pos, const int64_t *__restrict__ tok_off, rs_params p,
-              int acc_cap, int32_t *__restrict__ argmax, int32_t *__restrict__ topk,
-              float *__restrict__ lse, float *__restrict__ p_tok, int32_t *__restrict__ acc_len,
+              int acc_cap, const int32_t *__restrict__ argmax, const int32_t *__restrict__ topk,
+              const float *__restrict__ lse, float *__restrict__ p_tok, int32_t *__restrict__ acc_len,
               int32_t *__restrict__ acc_nodes, int32_t *__restrict__ bonus, int32_t *__restrict__ winner,
               uint8_t *__restrict__ commit, float *__restrict__ scores, int32_t *__restrict__ status) {
     const int b = blockIdx.x;
@@ -250,52 +405,14 @@ accept_decide(const float *__restrict__ logits, int V, int nchunks, const VI *__
     __shared__ int s_bad;
     __shared__ int s_best;  // (depth << 16) | (0xffff - node)
 
-    // ---- row statistics (every row of the request): one warp per row ----
-    // the row's chunk candidates (<= 32 * kCandPerLane) are loaded once into
-    // registers, then beta rounds of a warp-wide "best after the previous
-    // winner" reduction run on them
-    const int ncand = nchunks * beta;
-    for (int lr = warp; lr < N; lr += kDecThreads / 32) {
-        const long long r = n0 + lr;
-        MS ms{-INFINITY, 0.f};
-        for (int c = lane; c < nchunks; c += 32) ms = ms_merge(ms, part[r * nchunks + c]);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            MS u{__shfl_xor_sync(0xffffffffu, ms.m, o), __shfl_xor_sync(0xffffffffu, ms.s, o)};
-            ms = ms_merge(ms, u);
+    // ---- row statistics of the request's rows (written by accept_merge) ----
+    if (N <= RS_MAX_NODES) {
+        for (int lr = tid; lr < N; lr += kDecThreads) {
+            s_arg[lr] = argmax[n0 + lr];
+            s_lse[lr] = lse[n0 + lr];
         }
-        const float l = ms.s > 0.f ? ms.m + __logf(ms.s) : -INFINITY;
-        VI cv[kCandPerLane];
-#pragma unroll
-        for (int q = 0; q < kCandPerLane; ++q) {
-            const int c = lane + 32 * q;
-            cv[q] = c < ncand ? cand[r * ncand + c] : VI{-INFINITY, kNoId};
-        }
-        VI prev{INFINITY, -1};
-        for (int k = 0; k < beta; ++k) {
-            VI best{-INFINITY, kNoId};
-#pragma unroll
-            for (int q = 0; q < kCandPerLane; ++q) {
-                const VI x = cv[q];
-                if (x.i != kNoId && vi_before(prev.v, prev.i, x.v, x.i) && vi_before(x.v, x.i, best.v, best.i))
-                    best = x;
-            }
-            best = warp_vi_best(best);
-            prev = best;
-            if (lane == 0) {
-                const int id = best.i == kNoId ? -1 : best.i;
-                topk[r * beta + k] = id;
-                if (lr < RS_MAX_NODES) s_top[lr * RS_MAX_BETA + k] = id;
-                if (k == 0) {
-                    argmax[r] = id;
-                    lse[r] = l;
-                    if (lr < RS_MAX_NODES) {
-                        s_arg[lr] = id;
-                        s_lse[lr] = l;
-                    }
-                }
-            }
-        }
+        for (int x = tid; x < N * beta; x += kDecThreads)
+            s_top[(x / beta) * RS_MAX_BETA + (x % beta)] = topk[(long long)n0 * beta + x];
     }
 
     // ---- tree layout check ----
@@ -484,8 +601,8 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
                                const int32_t *tokens, const int32_t *parents, const uint8_t *source,
                                const int8_t *chain, const int32_t *sel_pos, const int64_t *tok_off,
                                rs_params p, int acc_cap, int32_t *argmax, int32_t *topk, float *lse,
-                               float *p_tok, int32_t *acc_len, int32_t *acc_nodes, int32_t *bonus,
-                               int32_t *winner, uint8_t *commit, float *scores, int32_t *status,
+                               float *p_tok, float *entropy, int32_t *acc_len, int32_t *acc_nodes,
+                               int32_t *bonus, int32_t *winner, uint8_t *commit, float *scores, int32_t *status,
                                void *workspace, size_t workspace_bytes, void *stream) {
     clear_error();
     RS_CHECK_ARG(R >= 0 && B >= 0, "rs_accept: negative size (R=%d, B=%d)", R, B);
@@ -520,20 +637,48 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
     VI *cand = cv.take<VI>((size_t)R * nchunks * p.beta);
     MS *part = cv.take<MS>((size_t)R * nchunks);
     if (R > 0) {
-        long long blocks = (long long)R * nchunks;
+        const long long blocks = (long long)R * nchunks;
         RS_CHECK_ARG(blocks < (1ll << 31), "rs_accept: R*chunks too large");
-        bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
-        if (vec)
-            accept_rows<true><<<(unsigned)blocks, kAccThreads, 0, st>>>(logits, V, nchunks, p.beta, cand, part);
+        const bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
+        const bool ent = entropy != nullptr;
+        const unsigned grid = (unsigned)std::min<long long>(blocks, 3ll * num_sms());
+        static int attr_done[64] = {0};
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+            cudaError_t e = cudaSuccess;
+            const int bytes = (int)kRowsSmem;
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(accept_rows<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(accept_rows<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(accept_rows<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(accept_rows<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+            if (e != cudaSuccess) {
+                set_error("rs_accept: cudaFuncSetAttribute: %s", cudaGetErrorString(e));
+                return RS_ERR_CUDA;
+            }
+            attr_done[dev] = 1;
+        }
+        if (vec && ent)
+            accept_rows<true, true><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, blocks, cand, part);
+        else if (vec)
+            accept_rows<true, false><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, blocks, cand, part);
+        else if (ent)
+            accept_rows<false, true><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, blocks, cand, part);
         else
-            accept_rows<false><<<(unsigned)blocks, kAccThreads, 0, st>>>(logits, V, nchunks, p.beta, cand, part);
+            accept_rows<false, false><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, blocks, cand, part);
         RS_CHECK_LAUNCH("rs_accept/accept_rows");
+        accept_merge<<<(R + kMergeThreads / 32 - 1) / (kMergeThreads / 32), kMergeThreads, 0, st>>>(
+            cand, part, nchunks, p.beta, R, argmax, topk, lse, entropy);
+        RS_CHECK_LAUNCH("rs_accept/accept_merge");
     }
     if (B > 0) {
-        accept_decide<<<B, kDecThreads, 0, st>>>(logits, V, nchunks, cand, part, node_off, tokens, parents,
-                                                 source, chain, sel_pos, tok_off, p, acc_cap, argmax, topk,
-                                                 lse, p_tok, acc_len, acc_nodes, bonus, winner, commit,
-                                                 scores, status);
+        accept_decide<<<B, kDecThreads, 0, st>>>(logits, V, node_off, tokens, parents, source, chain, sel_pos,
+                                                 tok_off, p, acc_cap, argmax, topk, lse, p_tok, acc_len, acc_nodes,
+                                                 bonus, winner, commit, scores, status);
         RS_CHECK_LAUNCH("rs_accept/accept_decide");
     }
     return RS_OK;

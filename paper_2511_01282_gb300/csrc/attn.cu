@@ -82,8 +82,9 @@ attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_
 
 // Block c merges the split segment whose first piece is c's last piece.
 // Phase 1: one thread per row forms M = max_p m_p and the weights
-// e^(m_p - M) / sum_p e^(m_p - M) l_p in shared memory.  Phase 2: the block
-// sweeps (row, 4 head-dim columns) items with float4 loads of the partial O.
+// e^(m_p - M) / sum_p e^(m_p - M) l_p in shared memory.  Phase 2: each thread
+// owns 16 (row, 4 head-dim columns) items and, piece by piece, accumulates
+// their float4 partials (16 independent loads in flight per thread).
 constexpr int kCombThreads = 256;
 constexpr int kMaxPieces = 1024;
 constexpr int kFastPieces = 16;  // pieces whose weights fit the shared table
@@ -144,31 +145,44 @@ attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
             for (int p = 0; p < np; ++p) s_w[p][r] /= L;
     }
     __syncthreads();
-    // phase 2: outputs, four columns per item
+    // phase 2: outputs, four columns per item; each thread keeps kItems items
+    // in flight so the partial loads of different items overlap
+    constexpr int kItems = kBM * 32 / kCombThreads;  // 16: all (row, column quad) items of D = 128
     const int d4 = D / 4;
-    for (int x = threadIdx.x; x < rows * d4; x += kCombThreads) {
-        const int r = x / d4, q = x - r * d4;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int p = 0; p < np; ++p) {
-            const long long prow = (long long)s_slot[p] * kBM + r;
+    const int nitems = rows * d4;
+    float4 acc[kItems];
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int p = 0; p < np; ++p) {
+        const long long base = (long long)s_slot[p] * kBM;
+#pragma unroll
+        for (int k = 0; k < kItems; ++k) {
+            const int x = threadIdx.x + k * kCombThreads;
+            if (x >= nitems) continue;
+            const int r = x / d4, q = x - r * d4;
             float w;
             if (fast) {
                 w = s_w[p][r];
             } else {
-                const float m = a.part_m[prow];
+                const float m = a.part_m[base + r];
                 w = m == -INFINITY ? 0.f : __expf(m - s_M[r]) / s_L[r];
             }
-            if (w == 0.f) continue;
-            const float4 o = *reinterpret_cast<const float4 *>(a.part_o + prow * D + q * 4);
-            acc.x += w * o.x;
-            acc.y += w * o.y;
-            acc.z += w * o.z;
-            acc.w += w * o.w;
+            const float4 o = *reinterpret_cast<const float4 *>(a.part_o + (base + r) * D + q * 4);
+            acc[k].x += w * o.x;
+            acc[k].y += w * o.y;
+            acc[k].z += w * o.z;
+            acc[k].w += w * o.w;
         }
+    }
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) {
+        const int x = threadIdx.x + k * kCombThreads;
+        if (x >= nitems) continue;
+        const int r = x / d4, q = x - r * d4;
         const int rr = mtile * kBM + r;
         const int i = rr / G, h = kvh * G + (rr - i * G);
         const long long orow = (long long)(n0 + i) * a.Hq + h;
-        *reinterpret_cast<float4 *>(a.out + orow * D + q * 4) = acc;
+        *reinterpret_cast<float4 *>(a.out + orow * D + q * 4) = acc[k];
         if (q == 0) a.lse[orow] = s_M[r] + __logf(s_L[r]);
     }
 }

@@ -2,14 +2,16 @@
 // (Section 3.2.1, Eq. 1-3 and step 4; Algorithm 1 step 1).
 //
 // Kernel 1 (entropy_partial): one CTA per (row, 8192-logit chunk).  Each
-// thread streams 32 logits with 128-bit loads and forms, relative to its own
-// maximum m, s = sum e^(z-m) and w = sum e^(z-m) (z-m); the CTA merges the
-// triples with warp shuffles and writes one triple per chunk.  Row entropy
-// is then H = ln s - w / s for the merged triple (the log-sum-exp form of
-// -sum p ln p).
-// Kernel 2 (gate_finalize): one CTA per request merges its rows' chunk
-// triples, writes the row entropies, pushes the committed rows into the
-// history and evaluates H_k, C_k, k* and the trigger in fp64.
+// thread streams 32 logits with 128-bit loads; relative to its warp's
+// maximum m the warp forms s = sum e^(z-m) and w = sum e^(z-m) (z-m) (plain
+// shuffle sums), and one thread merges the eight warp triples into the
+// chunk's.  Row entropy is then H = ln s - w / s for the merged triple (the
+// log-sum-exp form of -sum p ln p).
+// Kernel 2 (entropy_merge): one warp per row merges its chunk triples into
+// the row entropy.  Kernel 3 (gate_push): one CTA per request pushes the
+// committed rows' entropies into the history and evaluates H_k, C_k, k* and
+// the trigger in fp64.  rs_entropy_gate_rows runs kernel 3 alone on row
+// entropies that rs_accept already produced from the same logits.
 #include <math.h>
 
 #include <mutex>
@@ -47,21 +49,10 @@ __device__ __forceinline__ Ent3 ent_shfl(Ent3 a, int o) {
     return b;
 }
 
-// One thread's triple over its kGateVpt values (-inf padded).
-__device__ __forceinline__ Ent3 ent_local(const float (&v)[kGateVpt]) {
-    float mx = -INFINITY;
-#pragma unroll
-    for (int i = 0; i < kGateVpt; ++i) mx = fmaxf(mx, v[i]);
-    Ent3 r{mx, 0.f, 0.f};
-    if (mx == -INFINITY) return r;
-#pragma unroll
-    for (int i = 0; i < kGateVpt; ++i) {
-        float d = fmaxf(v[i] - mx, -1e30f);  // -inf -> -1e30: e = 0, e*d = 0
-        float e = __expf(d);
-        r.s += e;
-        r.w = fmaf(e, d, r.w);
-    }
-    return r;
+__device__ __forceinline__ float ex2f_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
 }
 
 template <bool kVec>
@@ -102,32 +93,72 @@ entropy_partial(const float *__restrict__ logits, int V, int nchunks, Ent3 *__re
         }
     }
 
-    Ent3 t = ent_local(v);
+    // warp maximum as the common reference: the warp's triple is a plain sum
+    float mx = -INFINITY;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) t = ent_merge(t, ent_shfl(t, o));
+    for (int i = 0; i < kGateVpt; ++i) mx = fmaxf(mx, v[i]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    Ent3 t{mx, 0.f, 0.f};
+    if (mx != -INFINITY) {
+        constexpr float kL2E = 1.4426950408889634f;
+        float s4[4] = {0.f, 0.f, 0.f, 0.f}, w4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < kGateVpt; ++i) {
+            const float d = fmaxf(v[i] - mx, -1e30f);  // -inf -> -1e30: e = 0, e*d = 0
+            const float e = ex2f_approx(d * kL2E);
+            s4[i & 3] += e;
+            w4[i & 3] = fmaf(e, d, w4[i & 3]);
+        }
+        float ss = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+        float ww = (w4[0] + w4[1]) + (w4[2] + w4[3]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            ss += __shfl_xor_sync(0xffffffffu, ss, o);
+            ww += __shfl_xor_sync(0xffffffffu, ww, o);
+        }
+        t.s = ss;
+        t.w = ww;
+    }
     __shared__ Ent3 sw[kGateThreads / 32];
     if ((tid & 31) == 0) sw[tid >> 5] = t;
     __syncthreads();
-    if (tid < 32) {
-        t = tid < kGateThreads / 32 ? sw[tid] : Ent3{-INFINITY, 0.f, 0.f};
+    if (tid == 0) {
+        Ent3 a = sw[0];
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) t = ent_merge(t, ent_shfl(t, o));
-        if (tid == 0) part[blk] = t;
+        for (int w = 1; w < kGateThreads / 32; ++w) a = ent_merge(a, sw[w]);
+        part[blk] = a;
     }
 }
 
-constexpr int kFinRows = 512;  // rows staged in shared memory per pass
+constexpr int kMergeThreads = 256;
 
-__global__ void __launch_bounds__(256)
-gate_finalize(const Ent3 *__restrict__ part, int nchunks, const int32_t *__restrict__ row_off,
-              const uint8_t *__restrict__ row_commit, rs_params p, float *__restrict__ hist,
-              int32_t *__restrict__ hist_n, float *__restrict__ entropy, int32_t *__restrict__ k_star,
-              float *__restrict__ h_best, uint8_t *__restrict__ entropy_ok) {
+__global__ void __launch_bounds__(kMergeThreads)
+entropy_merge(const Ent3 *__restrict__ part, int nchunks, int R, float *__restrict__ entropy) {
+    const int lane = threadIdx.x & 31;
+    const long long r = (long long)blockIdx.x * (kMergeThreads / 32) + (threadIdx.x >> 5);
+    if (r >= R) return;
+    Ent3 t{-INFINITY, 0.f, 0.f};
+    for (int c = lane; c < nchunks; c += 32) t = ent_merge(t, part[r * nchunks + c]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t = ent_merge(t, ent_shfl(t, o));
+    if (lane == 0) entropy[r] = t.s > 0.f ? (__logf(t.s) - t.w / t.s) : 0.f;
+}
+
+// Per request: push the committed rows' entropies into the history (row
+// order), then Algorithm 1 step 1 in fp64 (k upward, strict '<').
+constexpr int kPushThreads = 256;
+constexpr int kPushRows = 1024;  // rows staged in shared memory per pass
+
+__global__ void __launch_bounds__(kPushThreads)
+gate_push(const float *__restrict__ entropy, const int32_t *__restrict__ row_off,
+          const uint8_t *__restrict__ row_commit, rs_params p, float *__restrict__ hist,
+          int32_t *__restrict__ hist_n, int32_t *__restrict__ k_star, float *__restrict__ h_best,
+          uint8_t *__restrict__ entropy_ok) {
     const int b = blockIdx.x;
     const int r0 = row_off[b], r1 = row_off[b + 1];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    __shared__ float s_ent[kFinRows];
-    __shared__ uint8_t s_com[kFinRows];
+    __shared__ float s_ent[kPushRows];
+    __shared__ uint8_t s_com[kPushRows];
     __shared__ float s_h[RS_MAX_L];
     __shared__ int s_n;
     const int l = p.l;
@@ -137,24 +168,15 @@ gate_finalize(const Ent3 *__restrict__ part, int nchunks, const int32_t *__restr
         s_n = n;
         for (int i = 0; i < l; ++i) s_h[i] = hist[(long long)b * l + i];
     }
-    for (int base = r0; base < r1; base += kFinRows) {
-        const int rows = min(kFinRows, r1 - base);
-        // row entropies: one warp per row, lanes over chunks
-        for (int lr = warp; lr < rows; lr += blockDim.x >> 5) {
-            const long long r = base + lr;
-            Ent3 t{-INFINITY, 0.f, 0.f};
-            for (int c = lane; c < nchunks; c += 32) t = ent_merge(t, part[r * nchunks + c]);
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) t = ent_merge(t, ent_shfl(t, o));
-            if (lane == 0) {
-                const float e = t.s > 0.f ? (__logf(t.s) - t.w / t.s) : 0.f;
-                entropy[r] = e;
-                s_ent[lr] = e;
-            }
+    for (int base = r0; base < r1; base += kPushRows) {
+        const int rows = min(kPushRows, r1 - base);
+        __syncthreads();  // the previous pass is consumed
+        for (int lr = threadIdx.x; lr < rows; lr += kPushThreads) {
+            s_com[lr] = row_commit[base + lr];
+            s_ent[lr] = entropy[base + lr];
         }
-        for (int lr = threadIdx.x; lr < rows; lr += blockDim.x) s_com[lr] = row_commit[base + lr];
         __syncthreads();
-        if (threadIdx.x == 0) {  // push the committed rows, in row order
+        if (threadIdx.x == 0) {
             int n = s_n;
             for (int lr = 0; lr < rows; ++lr) {
                 if (!s_com[lr]) continue;
@@ -167,14 +189,12 @@ gate_finalize(const Ent3 *__restrict__ part, int nchunks, const int32_t *__restr
             }
             s_n = n;
         }
-        __syncthreads();
     }
     if (threadIdx.x != 0) return;
     const int n = s_n;
     for (int i = 0; i < l; ++i) hist[(long long)b * l + i] = s_h[i];
     hist_n[b] = n;
 
-    // Algorithm 1 step 1 in fp64: k upward, strict '<'
     double c_min = INFINITY, best = INFINITY;
     int kbest = 0;
     for (int k = 1; k <= n; ++k) {
@@ -191,6 +211,35 @@ gate_finalize(const Ent3 *__restrict__ part, int nchunks, const int32_t *__restr
     k_star[b] = kbest;
     h_best[b] = (float)best;
     entropy_ok[b] = (uint8_t)(kbest > 0 && best <= (double)p.theta_entropy);
+}
+
+// The three launches of a gate call over the chunk triples in `part`.
+rs_status launch_gate(const char *who, const float *logits, int R, int V, int nchunks, Ent3 *part,
+                      const int32_t *row_off, const uint8_t *row_commit, int B, rs_params p, float *hist,
+                      int32_t *hist_n, float *entropy, int32_t *k_star, float *h_best, uint8_t *entropy_ok,
+                      cudaStream_t st) {
+    if (R > 0) {
+        const long long blocks = (long long)R * nchunks;
+        if (blocks >= (1ll << 31)) {
+            set_error("%s: R*chunks too large", who);
+            return RS_ERR_INVALID_ARG;
+        }
+        const bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
+        if (vec)
+            entropy_partial<true><<<(unsigned)blocks, kGateThreads, 0, st>>>(logits, V, nchunks, part);
+        else
+            entropy_partial<false><<<(unsigned)blocks, kGateThreads, 0, st>>>(logits, V, nchunks, part);
+        RS_CHECK_LAUNCH(who);
+        entropy_merge<<<(R + kMergeThreads / 32 - 1) / (kMergeThreads / 32), kMergeThreads, 0, st>>>(
+            part, nchunks, R, entropy);
+        RS_CHECK_LAUNCH(who);
+    }
+    if (B > 0) {
+        gate_push<<<B, kPushThreads, 0, st>>>(entropy, row_off, row_commit, p, hist, hist_n, k_star, h_best,
+                                              entropy_ok);
+        RS_CHECK_LAUNCH(who);
+    }
+    return RS_OK;
 }
 
 }  // namespace
@@ -224,26 +273,10 @@ extern "C" rs_status rs_entropy_gate(const float *logits, int R, int V, const in
         set_error("rs_entropy_gate: workspace %zu bytes < %zu required", workspace_bytes, need);
         return RS_ERR_CAPACITY;
     }
-    cudaStream_t st = (cudaStream_t)stream;
     Carve cv(workspace);
     Ent3 *part = cv.take<Ent3>((size_t)R * nchunks);
-
-    if (R > 0) {
-        long long blocks = (long long)R * nchunks;
-        RS_CHECK_ARG(blocks < (1ll << 31), "rs_entropy_gate: R*chunks too large");
-        bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
-        if (vec)
-            entropy_partial<true><<<(unsigned)blocks, kGateThreads, 0, st>>>(logits, V, nchunks, part);
-        else
-            entropy_partial<false><<<(unsigned)blocks, kGateThreads, 0, st>>>(logits, V, nchunks, part);
-        RS_CHECK_LAUNCH("rs_entropy_gate/entropy_partial");
-    }
-    if (B > 0) {
-        gate_finalize<<<B, 256, 0, st>>>(part, nchunks, row_off, row_commit, p, hist, hist_n, entropy,
-                                         k_star, h_best, entropy_ok);
-        RS_CHECK_LAUNCH("rs_entropy_gate/gate_finalize");
-    }
-    return RS_OK;
+    return launch_gate("rs_entropy_gate", logits, R, V, nchunks, part, row_off, row_commit, B, p, hist, hist_n,
+                       entropy, k_star, h_best, entropy_ok, (cudaStream_t)stream);
 }
 
 // ============================================================ no-allocation variant
@@ -307,19 +340,21 @@ extern "C" rs_status rs_entropy_gate_noalloc(const float *logits, int R, int V, 
         if (!rs_last_error()[0]) set_error("rs_entropy_gate_noalloc: device %d not supported", dev);
         return RS_ERR_CUDA;
     }
-    cudaStream_t st = (cudaStream_t)stream;
-    if (R > 0) {
-        bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
-        if (vec)
-            entropy_partial<true><<<(unsigned)partials, kGateThreads, 0, st>>>(logits, V, nchunks, part);
-        else
-            entropy_partial<false><<<(unsigned)partials, kGateThreads, 0, st>>>(logits, V, nchunks, part);
-        RS_CHECK_LAUNCH("rs_entropy_gate_noalloc/entropy_partial");
-    }
-    if (B > 0) {
-        gate_finalize<<<B, 256, 0, st>>>(part, nchunks, row_off, row_commit, p, hist, hist_n, entropy, k_star,
-                                         h_best, entropy_ok);
-        RS_CHECK_LAUNCH("rs_entropy_gate_noalloc/gate_finalize");
-    }
+    return launch_gate("rs_entropy_gate_noalloc", logits, R, V, nchunks, part, row_off, row_commit, B, p, hist,
+                       hist_n, entropy, k_star, h_best, entropy_ok, (cudaStream_t)stream);
+}
+
+extern "C" rs_status rs_entropy_gate_rows(const float *entropy, const int32_t *row_off, const uint8_t *row_commit,
+                                          int B, rs_params p, float *hist, int32_t *hist_n, int32_t *k_star,
+                                          float *h_best, uint8_t *entropy_ok, void *stream) {
+    clear_error();
+    RS_CHECK_ARG(B >= 0, "rs_entropy_gate_rows: negative B");
+    RS_CHECK_ARG(p.l >= 1 && p.l <= RS_MAX_L, "rs_entropy_gate_rows: l=%d outside [1, %d]", p.l, RS_MAX_L);
+    RS_CHECK_ARG(B == 0 || (entropy && row_off && row_commit && hist && hist_n && k_star && h_best && entropy_ok),
+                 "rs_entropy_gate_rows: null pointer");
+    if (B == 0) return RS_OK;
+    gate_push<<<B, kPushThreads, 0, (cudaStream_t)stream>>>(entropy, row_off, row_commit, p, hist, hist_n, k_star,
+                                                            h_best, entropy_ok);
+    RS_CHECK_LAUNCH("rs_entropy_gate_rows");
     return RS_OK;
 }

@@ -4,8 +4,10 @@
 per-call workspaces, all plain torch allocations) and enqueues, on one
 stream, the calls of one step of Algorithm 1 in their data-flow order:
 
-    rs_entropy_gate -> rs_match_scan (keyed by k*, gated by the trigger)
-                    -> rs_tree_verify_attn -> rs_accept
+    trigger (rs_entropy_gate_rows on the row entropies of the last verify,
+             or rs_entropy_gate on the logits)
+      -> rs_match_scan (keyed by k*, gated by the trigger)
+      -> rs_tree_verify_attn -> rs_accept (also emits the row entropies)
 
 It computes nothing itself.  Inputs come as host numpy arrays (bf16 as
 uint16 bit patterns) with the layouts ``include/respec.h`` documents.
@@ -57,7 +59,8 @@ class VerifyStep:
             attn_out=z((R, Hq, D), torch.float32), attn_lse=z((R, Hq), torch.float32),
             attn_status=z(B, torch.int32),
             argmax=z(R, torch.int32), topk=z((R, p.beta), torch.int32), lse=z(R, torch.float32),
-            p_tok=z(R, torch.float32), acc_len=z(B, torch.int32), acc_nodes=z((B, acc_cap), torch.int32),
+            p_tok=z(R, torch.float32), acc_entropy=z(R, torch.float32),
+            acc_len=z(B, torch.int32), acc_nodes=z((B, acc_cap), torch.int32),
             bonus=z(B, torch.int32), winner=z(B, torch.int32), commit=z(R, torch.uint8),
             acc_status=z(B, torch.int32))
         self.ws = dict(
@@ -72,6 +75,13 @@ class VerifyStep:
         rs.rs_entropy_gate(d["logits"], self.R, self.V, d["row_off"], d["row_commit"], self.B, self.p,
                            d["hist"], d["hist_n"], o["entropy"], o["k_star"], o["h_best"],
                            o["entropy_ok"], self.ws["gate"], stream)
+
+    def gate_rows(self, stream=None):
+        """The trigger from the row entropies the last accept produced."""
+        d, o = self.d, self.out
+        rs.rs_entropy_gate_rows(o["acc_entropy"], d["row_off"], d["row_commit"], self.B, self.p,
+                                d["hist"], d["hist_n"], o["k_star"], o["h_best"], o["entropy_ok"],
+                                stream)
 
     def scan(self, k_star=None, gate_ok="gate", stream=None):
         d, o = self.d, self.out
@@ -88,20 +98,36 @@ class VerifyStep:
                                self.scale, o["attn_out"], o["attn_lse"], o["attn_status"],
                                self.ws["attn"], stream)
 
-    def accept(self, sel_pos=None, stream=None):
+    def accept(self, sel_pos=None, entropy=True, stream=None):
         d, o = self.d, self.out
         sp = d["sel_pos"] if sel_pos is None else sel_pos
         rs.rs_accept(d["logits"], self.R, self.V, d["node_off"], self.B, d["tree_tokens"], d["parents"],
                      d["source"], d["chain"], sp, d["tok_off"], self.p, self.acc_cap, o["argmax"],
-                     o["topk"], o["lse"], o["p_tok"], o["acc_len"], o["acc_nodes"], o["bonus"],
-                     o["winner"], o["commit"], d["scores"], o["acc_status"], self.ws["accept"], stream)
+                     o["topk"], o["lse"], o["p_tok"], o["acc_entropy"] if entropy else None,
+                     o["acc_len"], o["acc_nodes"], o["bonus"], o["winner"], o["commit"], d["scores"],
+                     o["acc_status"], self.ws["accept"], stream)
 
-    def step(self, stream=None):
-        """One pass of the whole hot path (4 calls, 9 kernel launches)."""
-        self.gate(stream)
+    def step(self, stream=None, fused=True):
+        """One pass of the whole hot path.
+
+        fused=True (steady state): the trigger uses the row entropies that the
+        previous step's rs_accept computed over the verify logits, so the
+        logits are read once per step; call prime() once first.
+        fused=False: rs_entropy_gate reads the logits itself.
+        """
+        if fused:
+            self.gate_rows(stream)
+        else:
+            self.gate(stream)
         self.scan(stream=stream)
         self.attn(stream)
         self.accept(stream=stream)
+
+    def prime(self, stream=None):
+        """Row entropies for the first fused step (one rs_accept pass)."""
+        scores = self.d["scores"].clone()
+        self.accept(stream=stream)
+        self.d["scores"].copy_(scores)
 
     # ------------------------------------------------------ host round trip
     def upload(self, stream=None):

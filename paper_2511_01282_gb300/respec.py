@@ -63,8 +63,9 @@ _SIGS = {
                                       C.c_size_t, _P]),
     "rs_accept_workspace_size": (C.c_size_t, [C.c_int, C.c_int, C.c_int]),
     "rs_accept": (C.c_int, [_P, C.c_int, C.c_int, _P, C.c_int, _P, _P, _P, _P, _P, _P, rs_params,
-                            C.c_int, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, C.c_size_t,
+                            C.c_int, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, C.c_size_t,
                             _P]),
+    "rs_entropy_gate_rows": (C.c_int, [_P, _P, _P, C.c_int, rs_params, _P, _P, _P, _P, _P, _P]),
 }
 
 
@@ -187,11 +188,18 @@ def rs_accept_workspace_size(R, V, beta):
 
 
 def rs_accept(logits, R, V, node_off, B, tokens, parents, source, chain, sel_pos, tok_off, p,
-              acc_cap, argmax, topk, lse, p_tok, acc_len, acc_nodes, bonus, winner, commit,
+              acc_cap, argmax, topk, lse, p_tok, entropy, acc_len, acc_nodes, bonus, winner, commit,
               scores, status, workspace, stream=None):
     wp, wb = _ws(workspace)
     _check(lib().rs_accept(_ptr(logits), R, V, _ptr(node_off), B, _ptr(tokens), _ptr(parents),
                            _ptr(source), _ptr(chain), _ptr(sel_pos), _ptr(tok_off), p, acc_cap,
-                           _ptr(argmax), _ptr(topk), _ptr(lse), _ptr(p_tok), _ptr(acc_len),
-                           _ptr(acc_nodes), _ptr(bonus), _ptr(winner), _ptr(commit),
-                           _ptr(scores), _ptr(status), wp, wb, _stream(stream)))
+                           _ptr(argmax), _ptr(topk), _ptr(lse), _ptr(p_tok), _ptr(entropy),
+                           _ptr(acc_len), _ptr(acc_nodes), _ptr(bonus), _ptr(winner),
+                           _ptr(commit), _ptr(scores), _ptr(status), wp, wb, _stream(stream)))
+
+
+def rs_entropy_gate_rows(entropy, row_off, row_commit, B, p, hist, hist_n, k_star, h_best,
+                         entropy_ok, stream=None):
+    _check(lib().rs_entropy_gate_rows(_ptr(entropy), _ptr(row_off), _ptr(row_commit), B, p,
+                                      _ptr(hist), _ptr(hist_n), _ptr(k_star), _ptr(h_best),
+                                      _ptr(entropy_ok), _stream(stream)))

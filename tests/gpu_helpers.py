@@ -144,6 +144,10 @@ def check_accept(w, st, acc_cap=None):
         a, b = host(o[k_gpu]), ref[k_ref]
         assert a.shape == b.shape and (a == b).all(), "accept %s differs" % k_gpu
     assert (host(st.d["scores"]) == ref["scores"]).all(), "updated scores differ"
+    # the row entropies of the same pass (rs_accept's fused output)
+    H = oracle.entropy_rows(w.logits)
+    err = np.max(np.abs(host(o["acc_entropy"]).astype(np.float64) - H)) if H.size else 0.0
+    assert err <= ENT_TOL, "accept entropy error %g nats" % err
     lse = host(o["lse"]).astype(np.float64)
     assert np.allclose(lse, ref["lse"], rtol=LSE_REL, atol=1e-6)
     # p(token) = exp(z - lse(parent row)): an lse within its relative bound
@@ -158,3 +162,22 @@ def check_accept(w, st, acc_cap=None):
                 tol[i] = LSE_REL * max(1.0, abs(ref["lse"][par]))
     assert (np.abs(pt - ref["p_tok"]) <= tol * ref["p_tok"] + 1e-7).all()
     return ref
+
+
+# ------------------------------------------------------------------ gate from rows
+def check_gate_rows(w, st):
+    """rs_entropy_gate_rows on rs_accept's entropies: bit-exact trigger."""
+    s = w.spec
+    st.d["hist"].copy_(torch.from_numpy(w.hist))
+    st.d["hist_n"].copy_(torch.from_numpy(w.hist_n))
+    st.gate_rows()
+    torch.cuda.synchronize()
+    o = st.out
+    H = host(o["acc_entropy"]).astype(np.float64)
+    g = oracle.gate(H, w.node_off, w.row_commit, w.hist, w.hist_n, s.l, f32(s.lambda_e),
+                    f32(s.theta_entropy))
+    assert (host(o["k_star"]) == g["k_star"]).all()
+    assert (host(o["entropy_ok"]) == g["ok"]).all()
+    assert (host(o["h_best"]) == g["h_best"].astype(np.float32)).all()
+    assert (host(st.d["hist"]) == g["hist"].astype(np.float32)).all()
+    assert (host(st.d["hist_n"]) == g["hist_n"]).all()

@@ -85,11 +85,11 @@ def test_bad_arguments_fail_before_launch(rs):
     st = L.rs_entropy_gate(f, 4, 100000, f, f, 1, p, f, f, f, f, f, f, f, 8, None)
     assert st == rs.RS_ERR_CAPACITY and "workspace" in rs.rs_last_error()
     # rs_accept: beta above V, negative tau, null pointers
-    st = L.rs_accept(f, 1, 3, f, 1, f, f, f, f, f, f, rs.params(beta=5), 4, *([f] * 11), f, 1 << 20, None)
+    st = L.rs_accept(f, 1, 3, f, 1, f, f, f, f, f, f, rs.params(beta=5), 4, *([f] * 12), f, 1 << 20, None)
     assert st == rs.RS_ERR_INVALID_ARG
-    st = L.rs_accept(f, 1, 30, f, 1, f, f, f, f, f, f, rs.params(tau=-1.0), 4, *([f] * 11), f, 1 << 20, None)
+    st = L.rs_accept(f, 1, 30, f, 1, f, f, f, f, f, f, rs.params(tau=-1.0), 4, *([f] * 12), f, 1 << 20, None)
     assert st == rs.RS_ERR_INVALID_ARG
-    st = L.rs_accept(None, 1, 30, f, 1, f, f, f, f, f, f, p, 4, *([f] * 11), f, 1 << 20, None)
+    st = L.rs_accept(None, 1, 30, f, 1, f, f, f, f, f, f, p, 4, *([f] * 12), f, 1 << 20, None)
     assert st == rs.RS_ERR_INVALID_ARG and "null" in rs.rs_last_error()
     # rs_match_scan: top_c above the limit, span_len 0
     st = L.rs_match_scan(f, f, 1, f, None, f, rs.params(top_c=9), 4, *([f] * 7), None, 0, None)

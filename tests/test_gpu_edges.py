@@ -106,6 +106,17 @@ def test_unaligned_and_odd_logits():
     check_accept(w, st)
 
 
+def test_accept_without_entropy_output():
+    w = synth.build(synth.small_spec(B=3, V=5000), seed=15)
+    st = make_step(w)
+    st.out["acc_entropy"].fill_(-5.0)
+    st.accept(entropy=False)
+    torch.cuda.synchronize()
+    assert (host(st.out["acc_entropy"]) == -5.0).all()  # untouched
+    st.d["scores"].copy_(torch.from_numpy(w.scores))
+    check_accept(w, st)
+
+
 def test_scan_truncation_and_skips():
     w = synth.build(synth.small_spec(B=4, repeat_prob=0.9, seg_len=(2, 4), V=50), seed=13)
     st = make_step(w)
@@ -145,29 +156,43 @@ def test_gate_with_empty_row_ranges():
 
 
 def test_cuda_graph_replay_matches_eager():
+    # the fused step (trigger on the previous accept's row entropies) and the
+    # unfused one, each captured once and replayed: same outputs as eager
     w = synth.make("tiny")
-    st = make_step(w)
-    st.step()
-    torch.cuda.synchronize()
-    eager = {k: host(v).copy() for k, v in st.out.items()}
-    st.reset_state()
-    s = torch.cuda.Stream()
-    s.wait_stream(torch.cuda.current_stream())
-    g = torch.cuda.CUDAGraph()
-    with torch.cuda.stream(s):
-        st.step(stream=s)  # warm the stream once outside the capture
-    torch.cuda.synchronize()
-    st.reset_state()
-    with torch.cuda.graph(g, stream=s):
-        st.step(stream=s)
-    st.reset_state()
-    for v in st.out.values():
-        v.fill_(-3)  # the replay has to rewrite every output
-    torch.cuda.synchronize()
-    n0 = rs.rs_launch_count()
-    with torch.cuda.stream(s):
-        g.replay()
-    torch.cuda.synchronize()
-    assert rs.rs_launch_count() == n0  # replays do not go through the host entry points
-    for k, v in eager.items():
-        assert (host(st.out[k]) == v).all(), k
+    for fused in (True, False):
+        st = make_step(w)
+        st.prime()
+        torch.cuda.synchronize()
+        carried = st.out["acc_entropy"].clone()  # the fused trigger's input
+        st.step(fused=fused)
+        torch.cuda.synchronize()
+        skip = {"acc_entropy"} | ({"entropy"} if fused else set())
+        eager = {k: host(v).copy() for k, v in st.out.items() if k not in skip}
+
+        def reset():
+            st.reset_state()
+            st.out["acc_entropy"].copy_(carried)
+
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        g = torch.cuda.CUDAGraph()
+        reset()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(s):
+            st.step(stream=s, fused=fused)  # warm the stream once outside the capture
+        torch.cuda.synchronize()
+        reset()
+        torch.cuda.synchronize()
+        with torch.cuda.graph(g, stream=s):
+            st.step(stream=s, fused=fused)
+        reset()
+        for k in eager:
+            st.out[k].fill_(-3)  # the replay has to rewrite every output
+        torch.cuda.synchronize()
+        n0 = rs.rs_launch_count()
+        with torch.cuda.stream(s):
+            g.replay()
+        torch.cuda.synchronize()
+        assert rs.rs_launch_count() == n0  # replays do not go through the host entry points
+        for k, v in eager.items():
+            assert (host(st.out[k]) == v).all(), (fused, k)

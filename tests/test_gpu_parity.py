@@ -11,7 +11,8 @@ import pytest
 import torch
 
 import synth
-from gpu_helpers import (check_accept, check_attn, check_gate, check_scan, make_step, sample_rows)
+from gpu_helpers import (check_accept, check_attn, check_gate, check_gate_rows, check_scan, make_step,
+                         sample_rows)
 
 pytestmark = pytest.mark.gpu
 
@@ -30,6 +31,7 @@ def _all_checks(w, attn_rows=None):
     check_scan(w, st, k_star=g["k_star"], gate_ok=g["ok"])  # keyed and gated by the trigger
     check_attn(w, st, rows=attn_rows)
     check_accept(w, st)
+    check_gate_rows(w, st)                                  # trigger on rs_accept's entropies
     return st
 
 
