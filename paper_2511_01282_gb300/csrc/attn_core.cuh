@@ -4,7 +4,9 @@
 // One CTA per SM walks its contiguous range of KV-tile units (see attn.cu).
 // Within a CTA, warps are specialised:
 //   warp 8 (1 thread)  TMA: K and V tiles of 128 keys x D into a 3-stage
-//                      ring of 128-byte-swizzled shared-memory buffers;
+//                      ring of 128-byte-swizzled shared-memory buffers (a
+//                      K slot is refilled once S of its tile is done, a V slot
+//                      once P V is);
 //   warp 9 (1 thread)  MMA: S = Q K^T into one of two TMEM buffers, then
 //                      O += P V with P read from TMEM (bf16, written over
 //                      S by the softmax warps) and V from shared memory;
@@ -46,7 +48,7 @@ constexpr int kTileBytes = kBN * 128 * 2;          // one 128-key x 128-dim bf16
 constexpr int kSmemK = 0;
 constexpr int kSmemV = kSmemK + kNS * kTileBytes;
 constexpr int kSmemBar = kSmemV + kNS * kTileBytes;
-constexpr int kNumBars = 3 * kNS + 12;
+constexpr int kNumBars = 4 * kNS + 12;
 constexpr int kSmemMisc = kSmemBar + kNumBars * 8;  // tmem base, abort flag
 constexpr int kSmemPref = kSmemMisc + 16;
 constexpr int kAttnMaxB = 4096;
@@ -206,8 +208,8 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
     unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                             ~uintptr_t(1023));
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kSmemBar);
-    uint64_t *kfull = bars, *vfull = bars + kNS, *kvempty = bars + 2 * kNS;
-    uint64_t *sfull = bars + 3 * kNS, *pfull = sfull + 2, *odone = pfull + 2, *qready = odone + 2;
+    uint64_t *kfull = bars, *vfull = bars + kNS, *kempty = bars + 2 * kNS, *vempty = bars + 3 * kNS;
+    uint64_t *sfull = bars + 4 * kNS, *pfull = sfull + 2, *odone = pfull + 2, *qready = odone + 2;
     uint64_t *ofree = qready + 1, *drain = ofree + 1;
     uint64_t *mxready = drain + 1, *lready = mxready + 2;  // softmax warpgroup exchanges
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + kSmemMisc);
@@ -219,7 +221,8 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
         for (int s = 0; s < kNS; ++s) {
             mbar_init(&kfull[s], 1);
             mbar_init(&vfull[s], 1);
-            mbar_init(&kvempty[s], 1);
+            mbar_init(&kempty[s], 1);
+            mbar_init(&vempty[s], 1);
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&sfull[s], 1);
@@ -261,14 +264,16 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                 const long long kv0 = a.kv_off[pc.b];
                 for (int jt = pc.j0; jt < pc.j1; ++jt, ++g) {
                     const int st = (int)(g % kNS);
-                    if (!(ok = mbar_wait(&kvempty[st], (uint32_t)(((g / kNS) & 1) ^ 1), s_abort, kWaitLimit)))
-                        break;
+                    const uint32_t free_par = (uint32_t)(((g / kNS) & 1) ^ 1);
                     const int row = (int)(kv0 + (long long)jt * kBN);
                     unsigned char *sk = smem + kSmemK + st * kTileBytes;
                     unsigned char *sv = smem + kSmemV + st * kTileBytes;
+                    // K is released as soon as S = Q K^T of the tile is done, V after P V
+                    if (!(ok = mbar_wait(&kempty[st], free_par, s_abort, kWaitLimit))) break;
                     mbar_expect_tx(&kfull[st], kTileTx);
 #pragma unroll
                     for (int kb = 0; kb < kKB; ++kb) tma_load_3d(sk + kb * 16384, &tmk, &kfull[st], kb * 64, pc.kvh, row);
+                    if (!(ok = mbar_wait(&vempty[st], free_par, s_abort, kWaitLimit))) break;
                     mbar_expect_tx(&vfull[st], kTileTx);
 #pragma unroll
                     for (int kb = 0; kb < kKB; ++kb) tma_load_3d(sv + kb * 16384, &tmv, &vfull[st], kb * 64, pc.kvh, row);
@@ -305,6 +310,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                     umma_ts(d_s, q_tm + kk * 8, sdesc_sw128(k_addr + off, 16, 1024), idS, kk > 0);
                 }
                 umma_commit(&sfull[gt & 1]);
+                umma_commit(&kempty[st]);
                 return true;
             };
             for (long long u = u0; u < u1 && ok; ++piece) {
@@ -329,7 +335,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                     for (int ks = 0; ks < kBN / 16; ++ks)
                         umma_ts(tmem + kTmO, p_tm + ks * 8, sdesc_sw128(v_addr + ks * 2048, 16384, 1024), idO,
                                 (tl > 0 || ks > 0) ? 1u : 0u);
-                    umma_commit(&kvempty[st]);
+                    umma_commit(&vempty[st]);
                     umma_commit(&odone[gt & 1]);
                 }
                 g += n;
