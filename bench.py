@@ -54,6 +54,27 @@ def parse():
     return ap.parse_args()
 
 
+# ------------------------------------------------------------------ ranks
+def rank_seed(seed, rank):
+    """Each rank draws its own batch (requests are independent: weak scaling)."""
+    return seed + 7919 * rank
+
+
+def slowest(value, dist, device):
+    """Max over ranks of a per-rank duration (identity without a process group)."""
+    if dist is None:
+        return float(value)
+    import torch
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(steps_per_rank, world, seconds):
+    """Whole-job throughput: every rank's steps over the slowest rank's time."""
+    return steps_per_rank * world / seconds
+
+
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -241,7 +262,7 @@ def run_ours(args, rank, world, local_rank):
     if args.requests:
         import dataclasses
         spec = dataclasses.replace(spec, B=min(args.requests, spec.B))
-    w = synth.build(spec, seed=args.seed + 7919 * rank)
+    w = synth.build(spec, seed=rank_seed(args.seed, rank))
     s = w.spec
     p = rs.params(**s.params())
     st = VerifyStep(arrays_from_workload(w), p, s.Hq, s.Hkv, s.D, pos_cap=s.pos_cap, pinned_host=True)
@@ -291,13 +312,9 @@ def run_ours(args, rank, world, local_rank):
     e1.record(stream)
     torch.cuda.synchronize()
     barrier()
-    t_ms = e0.elapsed_time(e1)
-    if dist is not None:
-        tt = torch.tensor([t_ms], device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t_ms = float(tt.item())
+    t_ms = slowest(e0.elapsed_time(e1), dist, "cuda")
     ms_per_step = t_ms / K
-    value = K * world / (t_ms / 1e3)
+    value = job_rate(K, world, t_ms / 1e3)
 
     # ---- per-call device time: a CUDA graph of n back-to-back calls, replayed
     # on the timed stream between two events (no host launch gaps inside)
@@ -340,10 +357,7 @@ def run_ours(args, rank, world, local_rank):
         stream.synchronize()
     e2e_s = time.perf_counter() - t0
     barrier()
-    if dist is not None:
-        tt = torch.tensor([e2e_s], device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_s = float(tt.item())
+    e2e_s = slowest(e2e_s, dist, "cuda")
     clocks.stop()
 
     peaks, peak_kind = load_peaks()
@@ -371,7 +385,7 @@ def run_ours(args, rank, world, local_rank):
                      "launch_ms": call_ms["attn"], "traffic": committed_traffic(args.workload),
                      "tflops": by["flops"] / attn_s / 1e12},
         "call_ms": call_ms,
-        "e2e": {"value": K * world / e2e_s, "unit": "steps/s", "h2d_bytes_per_step": h2d,
+        "e2e": {"value": job_rate(K, world, e2e_s), "unit": "steps/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches_per_step * K,
         "launches_per_step": launches_per_step,
