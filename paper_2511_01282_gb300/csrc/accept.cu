@@ -16,11 +16,12 @@
 // merges the lists).
 // No dynamic register indexing.
 // Kernel 2 (accept_merge): one warp per row merges the chunk results into
-// argmax, top-beta, log-sum-exp and (optionally) the row entropy.
+// argmax, top-beta, log-sum-exp, the row's largest logit (workspace, for
+// kernel 3) and (optionally) the row entropy.
 // Kernel 3 (accept_decide): one CTA per request checks the tree, verifies
-// model nodes (each thread walks its own root path), runs the look-ahead
-// procedure per chain (one thread per chain), picks the winner and updates
-// the scores.
+// model nodes (each thread walks its own root path over per-node match
+// flags), runs the look-ahead procedure per chain (one thread per chain),
+// picks the winner and updates the scores (one thread per selection).
 #include <math.h>
 
 #include <algorithm>
@@ -337,7 +338,7 @@ constexpr int kCandPerLane = 8;
 __global__ void __launch_bounds__(kMergeThreads)
 accept_merge(const VI *__restrict__ cand, const MS *__restrict__ part, int nchunks, int beta, int R,
              int32_t *__restrict__ argmax, int32_t *__restrict__ topk, float *__restrict__ lse,
-             float *__restrict__ entropy) {
+             float *__restrict__ entropy, float *__restrict__ rowmax) {
     const int lane = threadIdx.x & 31;
     const long long r = (long long)blockIdx.x * (kMergeThreads / 32) + (threadIdx.x >> 5);
     if (r >= R) return;
@@ -366,7 +367,10 @@ accept_merge(const VI *__restrict__ cand, const MS *__restrict__ part, int nchun
         if (lane == 0) {
             const int id = best.i == kNoId ? -1 : best.i;
             topk[r * beta + k] = id;
-            if (k == 0) argmax[r] = id;
+            if (k == 0) {
+                argmax[r] = id;
+                rowmax[r] = best.v;
+            }
         }
     }
     if (lane == 0) {
@@ -376,16 +380,27 @@ accept_merge(const VI *__restrict__ cand, const MS *__restrict__ part, int nchun
 }
 
 constexpr int kDecThreads = 512;
+constexpr int kNodeWords = RS_MAX_NODES / 32;
 
+// One CTA per request.  Every global read happens in two dependent rounds
+// at the start (the tree, the row statistics and the selected positions'
+// scores; then the logit of each node's token in its parent's row); the rest
+// works on shared memory.  Per node it precomputes the greedy match
+// (token == argmax of the parent row) and the relaxed check of Eq. 6-7
+// (token among the parent row's top beta and max logit - token logit <= tau
+// in fp64), so each chain's look-ahead walk and each model node's path check
+// read only flags.  Chain c's nodes are ranked by popcounts of per-chain
+// membership masks (one warp ballot per 32 nodes).
 __global__ void __launch_bounds__(kDecThreads)
 accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict__ node_off,
               const int32_t *__restrict__ tokens, const int32_t *__restrict__ parents,
               const uint8_t *__restrict__ source, const int8_t *__restrict__ chain,
               const int32_t *__restrict__ sel_pos, const int64_t *__restrict__ tok_off, rs_params p,
               int acc_cap, const int32_t *__restrict__ argmax, const int32_t *__restrict__ topk,
-              const float *__restrict__ lse, float *__restrict__ p_tok, int32_t *__restrict__ acc_len,
-              int32_t *__restrict__ acc_nodes, int32_t *__restrict__ bonus, int32_t *__restrict__ winner,
-              uint8_t *__restrict__ commit, float *__restrict__ scores, int32_t *__restrict__ status) {
+              const float *__restrict__ lse, const float *__restrict__ rowmax, float *__restrict__ p_tok,
+              int32_t *__restrict__ acc_len, int32_t *__restrict__ acc_nodes, int32_t *__restrict__ bonus,
+              int32_t *__restrict__ winner, uint8_t *__restrict__ commit, float *__restrict__ scores,
+              int32_t *__restrict__ status) {
     const int b = blockIdx.x;
     const int n0 = node_off[b];
     const int N = node_off[b + 1] - n0;
@@ -393,72 +408,125 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
     const int beta = p.beta, top_c = p.top_c;
 
     __shared__ int s_arg[RS_MAX_NODES];
-    __shared__ float s_lse[RS_MAX_NODES];
     __shared__ int s_top[RS_MAX_NODES * RS_MAX_BETA];
     __shared__ int s_par[RS_MAX_NODES];
     __shared__ int s_tok[RS_MAX_NODES];
+    __shared__ float s_zmax[RS_MAX_NODES];  // each row's largest logit
+    __shared__ float s_ztok[RS_MAX_NODES];  // node i: logit of its token in its parent's row
     __shared__ uint8_t s_src[RS_MAX_NODES];
     __shared__ int8_t s_chn[RS_MAX_NODES];
+    __shared__ uint8_t s_g[RS_MAX_NODES];   // greedy match
+    __shared__ uint8_t s_rx[RS_MAX_NODES];  // relaxed check (Eq. 6 and Eq. 7)
+    __shared__ uint32_t s_cmask[RS_MAX_TOPC][kNodeWords];
     __shared__ int s_cnodes[RS_MAX_TOPC][RS_MAX_NODES];
     __shared__ int s_clen[RS_MAX_TOPC];
     __shared__ int s_cacc[RS_MAX_TOPC];
-    __shared__ int s_bad;
+    __shared__ int s_selp[RS_MAX_TOPC];
+    __shared__ float s_selS[RS_MAX_TOPC];
+    __shared__ int s_bad, s_stt, s_win, s_dup;
     __shared__ int s_best;  // (depth << 16) | (0xffff - node)
 
-    // ---- row statistics of the request's rows (written by accept_merge) ----
-    if (N <= RS_MAX_NODES) {
-        for (int lr = tid; lr < N; lr += kDecThreads) {
-            s_arg[lr] = argmax[n0 + lr];
-            s_lse[lr] = lse[n0 + lr];
+    int st = 0;
+    if (N > RS_MAX_NODES) st = RS_ST_TOO_LARGE;
+    else if (N < 1) st = RS_ST_BAD_TREE;
+    if (tid == 0) {
+        s_bad = 0;
+        s_best = 0;
+        s_stt = 0;
+    }
+    const long long t0 = tok_off[b];
+    const long long t = tok_off[b + 1] - t0;
+    if (tid < top_c) {  // the selected positions and their scores (Eq. 4-5 inputs)
+        const int pos = sel_pos[(long long)b * top_c + tid];
+        s_selp[tid] = pos;
+        s_selS[tid] = (pos >= 0 && (long long)pos < t) ? scores[t0 + pos] : 0.f;
+    }
+    __syncthreads();
+
+    // ---- round 1 + 2: tree, row statistics, token logits ----
+    if (st == 0) {
+        for (int i = tid; i < N; i += kDecThreads) {
+            const int pa = parents[n0 + i];
+            const int sr = source[n0 + i];
+            const int ch = chain[n0 + i];
+            const int tk = tokens[n0 + i];
+            s_arg[i] = argmax[n0 + i];
+            s_zmax[i] = rowmax[n0 + i];
+            s_par[i] = pa;
+            s_tok[i] = tk;
+            s_src[i] = (uint8_t)sr;
+            s_chn[i] = (int8_t)ch;
+            commit[n0 + i] = 0;
+            bool bad;
+            if (i == 0) bad = (pa != -1 || sr != 0 || ch != -1);
+            else bad = (pa < 0 || pa >= i || sr < 1 || sr > 2 || (sr == 2 && (ch < 0 || ch >= top_c)) ||
+                        (sr == 1 && ch != -1) || tk < 0 || tk >= V);
+            if (bad) {
+                atomicOr(&s_bad, 1);
+            } else if (i == 0) {
+                p_tok[n0] = 1.f;
+            } else {
+                const float z = logits[(long long)(n0 + pa) * V + tk];
+                s_ztok[i] = z;
+                p_tok[n0 + i] = __expf(z - lse[n0 + pa]);
+            }
         }
         for (int x = tid; x < N * beta; x += kDecThreads)
             s_top[(x / beta) * RS_MAX_BETA + (x % beta)] = topk[(long long)n0 * beta + x];
     }
-
-    // ---- tree layout check ----
-    if (tid == 0) {
-        s_bad = 0;
-        s_best = 0;
-    }
     __syncthreads();
-    int st = 0;
-    if (N > RS_MAX_NODES) st = RS_ST_TOO_LARGE;
-    else if (N < 1) st = RS_ST_BAD_TREE;
-    if (st == 0) {
-        for (int i = tid; i < N; i += kDecThreads) {
-            int pa = parents[n0 + i];
-            int sr = source[n0 + i];
-            int ch = chain[n0 + i];
-            s_par[i] = pa;
-            s_tok[i] = tokens[n0 + i];
-            s_src[i] = (uint8_t)sr;
-            s_chn[i] = (int8_t)ch;
-            bool bad;
-            if (i == 0) bad = (pa != -1 || sr != 0 || ch != -1);
-            else bad = (pa < 0 || pa >= i || sr < 1 || sr > 2 || (sr == 2 && (ch < 0 || ch >= top_c)) ||
-                        (sr == 1 && ch != -1) || s_tok[i] < 0 || s_tok[i] >= V);
-            if (bad) atomicOr(&s_bad, 1);
+    const bool ok1 = st == 0 && s_bad == 0;
+
+    // ---- model nodes hang from the root or from model nodes; chain
+    // membership masks; per-node greedy and relaxed flags ----
+    if (ok1) {
+        for (int i = 1 + tid; i < N; i += kDecThreads) {
+            const int pa = s_par[i], x = s_tok[i];
+            if (s_src[i] == 1 && s_src[pa] > 1) atomicOr(&s_bad, 1);
+            s_g[i] = (uint8_t)(x == s_arg[pa]);
+            bool in_top = false;
+            for (int j = 0; j < beta; ++j) in_top |= (s_top[pa * RS_MAX_BETA + j] == x);
+            const double gap = (double)s_zmax[pa] - (double)s_ztok[i];
+            s_rx[i] = (uint8_t)(in_top && gap <= (double)p.tau);
         }
-        __syncthreads();
-        if (!s_bad) {
-            // model nodes hang from the root or from model nodes
-            for (int i = 1 + tid; i < N; i += kDecThreads)
-                if (s_src[i] == 1 && s_src[s_par[i]] > 1) atomicOr(&s_bad, 1);
-            // chain c: its nodes in index order form a path from the root
-            if (tid < top_c) {
-                int c = tid, L = 0, last = 0;
-                for (int i = 1; i < N; ++i) {
-                    if (s_src[i] != 2 || s_chn[i] != c) continue;
-                    if (s_par[i] != last) atomicOr(&s_bad, 1);
-                    s_cnodes[c][L++] = i;
-                    last = i;
-                }
-                s_clen[c] = L;
+        if (warp < kNodeWords) {
+            const int i = warp * 32 + lane;
+            const int ch = (i > 0 && i < N && s_src[i] == 2) ? s_chn[i] : -1;
+            for (int c = 0; c < top_c; ++c) {
+                const uint32_t m = __ballot_sync(0xffffffffu, ch == c);
+                if (lane == 0) s_cmask[c][warp] = m;
             }
         }
-        __syncthreads();
-        if (s_bad) st = RS_ST_BAD_TREE;
     }
+    __syncthreads();
+    const bool ok2 = ok1 && s_bad == 0;
+    // ---- chain c in index order: node of rank r ----
+    if (ok2) {
+        for (int i = 1 + tid; i < N; i += kDecThreads) {
+            if (s_src[i] != 2) continue;
+            const int c = s_chn[i], w = i >> 5;
+            int rank = __popc(s_cmask[c][w] & ((1u << (i & 31)) - 1u));
+            for (int q = 0; q < w; ++q) rank += __popc(s_cmask[c][q]);
+            s_cnodes[c][rank] = i;
+        }
+        if (tid < top_c) {
+            int L = 0;
+#pragma unroll
+            for (int q = 0; q < kNodeWords; ++q) L += __popc(s_cmask[tid][q]);
+            s_clen[tid] = L;
+        }
+    }
+    __syncthreads();
+    // ---- each chain is a path from the root: rank r hangs from rank r - 1 ----
+    if (ok2) {
+        for (int x = tid; x < top_c * RS_MAX_NODES; x += kDecThreads) {
+            const int c = x / RS_MAX_NODES, r = x - c * RS_MAX_NODES;
+            if (r >= s_clen[c]) continue;
+            if (s_par[s_cnodes[c][r]] != (r == 0 ? 0 : s_cnodes[c][r - 1])) atomicOr(&s_bad, 1);
+        }
+    }
+    __syncthreads();
+    if (st == 0 && s_bad) st = RS_ST_BAD_TREE;
 
     // ---- outputs of a rejected request ----
     if (st != 0) {
@@ -476,47 +544,29 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
         return;
     }
 
-    // ---- p_tok and strict verification of model nodes ----
-    for (int i = tid; i < N; i += kDecThreads) {
-        commit[n0 + i] = 0;
-        if (i == 0) {
-            p_tok[n0] = 1.f;
-            continue;
+    // ---- strict verification of model nodes: every node on the root path matches ----
+    for (int i = 1 + tid; i < N; i += kDecThreads) {
+        if (s_src[i] != 1) continue;
+        bool ok = true;
+        int depth = 0;
+        for (int a = i; a > 0; a = s_par[a]) {
+            ok = ok && s_g[a];
+            ++depth;
         }
-        int pa = s_par[i];
-        float z = logits[(long long)(n0 + pa) * V + s_tok[i]];
-        p_tok[n0 + i] = __expf(z - s_lse[pa]);
-        if (s_src[i] == 1) {
-            bool ok = true;
-            int depth = 0, a = i;
-            while (a > 0) {
-                ok = ok && (s_tok[a] == s_arg[s_par[a]]);
-                ++depth;
-                a = s_par[a];
-            }
-            if (ok) atomicMax(&s_best, (depth << 16) | (0xffff - i));
-        }
+        if (ok) atomicMax(&s_best, (depth << 16) | (0xffff - i));
     }
 
     // ---- relaxed verification with look-ahead, one thread per chain ----
     if (tid < top_c) {
         const int c = tid, L = s_clen[c];
         const int *d = s_cnodes[c];
-        auto greedy = [&](int j) { return s_tok[d[j]] == s_arg[s_par[d[j]]]; };
         int l0 = 0;
-        while (l0 < L && greedy(l0)) ++l0;
+        while (l0 < L && s_g[d[l0]]) ++l0;
         int cur = l0, last = l0;
         for (int att = 0; att < p.phi; ++att) {
-            if (cur >= L) break;
-            const int row = s_par[d[cur]];
-            const int x = s_tok[d[cur]];
-            bool in_top = false;
-            for (int j = 0; j < beta; ++j) in_top |= (s_top[row * RS_MAX_BETA + j] == x);
-            const float *zr = logits + (long long)(n0 + row) * V;
-            double gap = (double)zr[s_arg[row]] - (double)zr[x];
-            if (!(in_top && gap <= (double)p.tau)) break;
+            if (cur >= L || !s_rx[d[cur]]) break;
             int xi = 0;
-            while (cur + 1 + xi < L && greedy(cur + 1 + xi)) ++xi;
+            while (cur + 1 + xi < L && s_g[d[cur + 1 + xi]]) ++xi;
             if (xi >= p.m) {
                 last = cur + 1 + xi;
                 cur = last;
@@ -528,10 +578,10 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
     }
     __syncthreads();
 
-    // ---- winner, accepted path, bonus, commit, EMA ----
+    // ---- winner, accepted path, bonus, commit ----
     if (tid == 0) {
-        int model_len = s_best >> 16;
-        int best_node = model_len > 0 ? 0xffff - (s_best & 0xffff) : 0;
+        const int model_len = s_best >> 16;
+        const int best_node = model_len > 0 ? 0xffff - (s_best & 0xffff) : 0;
         int best_len = model_len, win = model_len > 0 ? -1 : -2;
         for (int c = 0; c < top_c; ++c)
             if (s_cacc[c] > best_len) {
@@ -550,7 +600,7 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
             }
         } else if (win >= 0) {
             for (int j = 0; j < best_len; ++j) {
-                int a = s_cnodes[win][j];
+                const int a = s_cnodes[win][j];
                 if (j < acc_cap) acc_nodes[(long long)b * acc_cap + j] = a;
                 commit[n0 + a] = 1;
                 last_node = a;
@@ -558,29 +608,48 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
         }
         for (int j = best_len; j < acc_cap; ++j) acc_nodes[(long long)b * acc_cap + j] = -1;
         commit[n0] = 1;
-        int stt = best_len > acc_cap ? RS_ST_TRUNCATED : 0;
         acc_len[b] = best_len;
         winner[b] = win;
         bonus[b] = s_arg[last_node];
+        s_win = win;
+        s_stt = best_len > acc_cap ? RS_ST_TRUNCATED : 0;
+        // a position selected twice is updated twice, in selection order
+        int dup = 0;
+        for (int c = 0; c < top_c; ++c)
+            for (int c2 = 0; c2 < c; ++c2)
+                dup |= (s_selp[c] >= 0 && s_selp[c] == s_selp[c2]);
+        s_dup = dup;
+    }
+    __syncthreads();
 
-        // Eq. 4-5 in fp64, rounded once to the fp32 table
-        const long long t0 = tok_off[b];
-        const long long t = tok_off[b + 1] - t0;
-        const double a = (double)p.alpha;
+    // ---- Eq. 4-5 in fp64, rounded once to the fp32 table ----
+    const double a = (double)p.alpha;
+    auto ema = [&](int c, double S) -> double {
+        const double R = (s_win == c) ? __ddiv_rn((double)s_cacc[c], (double)s_clen[c]) : 0.0;
+        return __dadd_rn(__dmul_rn(__dsub_rn(1.0, a), S), __dmul_rn(a, R));
+    };
+    if (!s_dup) {
+        if (tid < top_c) {
+            const int c = tid, pos = s_selp[c];
+            if (pos >= 0 && s_clen[c] != 0) {
+                if ((long long)pos >= t) atomicOr(&s_stt, RS_ST_BAD_POS);
+                else scores[t0 + pos] = __double2float_rn(ema(c, (double)s_selS[c]));
+            }
+        }
+    } else if (tid == 0) {
         for (int c = 0; c < top_c; ++c) {
-            int pos = sel_pos[(long long)b * top_c + c];
+            const int pos = s_selp[c];
             if (pos < 0 || s_clen[c] == 0) continue;
             if ((long long)pos >= t) {
-                stt |= RS_ST_BAD_POS;
+                s_stt |= RS_ST_BAD_POS;
                 continue;
             }
-            double R = (win == c) ? __ddiv_rn((double)s_cacc[c], (double)s_clen[c]) : 0.0;
             float *S = scores + t0 + pos;
-            double upd = __dadd_rn(__dmul_rn(__dsub_rn(1.0, a), (double)(*S)), __dmul_rn(a, R));
-            *S = __double2float_rn(upd);
+            *S = __double2float_rn(ema(c, (double)(*S)));
         }
-        status[b] = stt;
     }
+    __syncthreads();
+    if (tid == 0) status[b] = s_stt;
 }
 
 }  // namespace
@@ -594,6 +663,7 @@ extern "C" size_t rs_accept_workspace_size(int R, int V, int beta) {
     Carve cv(nullptr);
     cv.take<VI>((size_t)R * nchunks * beta);
     cv.take<MS>((size_t)R * nchunks);
+    cv.take<float>((size_t)R);
     return cv.used();
 }
 
@@ -636,6 +706,7 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
     Carve cv(workspace);
     VI *cand = cv.take<VI>((size_t)R * nchunks * p.beta);
     MS *part = cv.take<MS>((size_t)R * nchunks);
+    float *rowmax = cv.take<float>((size_t)R);
     if (R > 0) {
         const long long blocks = (long long)R * nchunks;
         RS_CHECK_ARG(blocks < (1ll << 31), "rs_accept: R*chunks too large");
@@ -672,12 +743,12 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
             accept_rows<false, false><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, blocks, cand, part);
         RS_CHECK_LAUNCH("rs_accept/accept_rows");
         accept_merge<<<(R + kMergeThreads / 32 - 1) / (kMergeThreads / 32), kMergeThreads, 0, st>>>(
-            cand, part, nchunks, p.beta, R, argmax, topk, lse, entropy);
+            cand, part, nchunks, p.beta, R, argmax, topk, lse, entropy, rowmax);
         RS_CHECK_LAUNCH("rs_accept/accept_merge");
     }
     if (B > 0) {
         accept_decide<<<B, kDecThreads, 0, st>>>(logits, V, node_off, tokens, parents, source, chain, sel_pos,
-                                                 tok_off, p, acc_cap, argmax, topk, lse, p_tok, acc_len, acc_nodes,
+                                                 tok_off, p, acc_cap, argmax, topk, lse, rowmax, p_tok, acc_len, acc_nodes,
                                                  bonus, winner, commit, scores, status);
         RS_CHECK_LAUNCH("rs_accept/accept_decide");
     }

@@ -16,7 +16,7 @@
 //   attn_prep validates each tree and builds a 256-bit ancestor set per
 //   node; the tree part of the mask is a bit test on it.
 // Launches: attn_prep (B CTAs) -> attn_tc_kernel (one CTA per SM; see
-// attn_core.cuh) -> attn_combine (one CTA per SM).
+// attn_core.cuh) -> attn_combine (four CTAs per range).
 #include <cudaTypedefs.h>
 #include <math.h>
 
@@ -80,21 +80,29 @@ attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_
     if (tid == 0) status[b] = st;
 }
 
-// Block c merges the split segment whose first piece is c's last piece.
-// Phase 1: one thread per row forms M = max_p m_p and the weights
-// e^(m_p - M) / sum_p e^(m_p - M) l_p in shared memory.  Phase 2: each thread
-// owns 16 (row, 4 head-dim columns) items and, piece by piece, accumulates
-// their float4 partials (16 independent loads in flight per thread).
+// Block (c, y) merges rows [32 y, 32 y + 32) of the split segment whose first
+// piece is c's last piece (four blocks per segment; the pieces are the
+// partials of the CTAs c .. c1 whose ranges cut the segment).
+// Phase 1: thread (row r, lane group j) folds the (m, l) pairs of pieces j,
+// j + 8, ... into a running (max, sum); warp 0 merges the eight folds into the
+// row's M = max_p m_p and 1 / L, L = sum_p e^(m_p - M) l_p.  Phase 2: each
+// thread owns D / 32 (row, 4 head-dim columns) items and sums e^(m_p - M) O_p
+// over the pieces, four pieces per round, so a round keeps 4 x D / 32 float4
+// partial loads and their m_p loads in flight.  The summation order is fixed
+// (piece order), so the result does not depend on timing.
 constexpr int kCombThreads = 256;
+constexpr int kCombRows = 32;                    // rows per block
+constexpr int kCombGroups = kBM / kCombRows;     // blocks per split segment
+constexpr int kCombFold = kCombThreads / kCombRows;  // lane groups in phase 1
+constexpr int kCombBatch = 4;                    // pieces per phase-2 round
 constexpr int kMaxPieces = 1024;
-constexpr int kFastPieces = 16;  // pieces whose weights fit the shared table
 
 __global__ void __launch_bounds__(kCombThreads)
 attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
     extern __shared__ int s_pref[];
     __shared__ int s_slot[kMaxPieces];
-    __shared__ float s_w[kFastPieces][kBM];
-    __shared__ float s_M[kBM], s_L[kBM];
+    __shared__ float s_fm[kCombFold][kCombRows], s_fl[kCombFold][kCombRows];
+    __shared__ float s_M[kCombRows], s_iL[kCombRows];
     __shared__ int s_np;
     unit_prefix(info, a.B, s_pref);
     const long long W = s_pref[a.B];
@@ -108,6 +116,13 @@ attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
     const long long seg_start = s_pref[b] + (long long)seg * ri.nt;
     const long long seg_end = seg_start + ri.nt;
     if (!(seg_start >= u0 && seg_end > u1)) return;  // not the first owner of a split segment
+    const int G = a.Hq / a.Hkv;
+    const int n0 = a.node_off[b];
+    const int N = a.node_off[b + 1] - n0;
+    const int kvh = seg / ri.mt, mtile = seg - kvh * ri.mt;
+    const int r0 = blockIdx.y * kCombRows;
+    const int rows = min(kCombRows, N * G - mtile * kBM - r0);
+    if (rows <= 0) return;
     const long long c1 = owner_of(seg_end - 1, W, Gc);
     if (threadIdx.x == 0) {
         int np = 0;
@@ -120,70 +135,101 @@ attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
     }
     __syncthreads();
     const int np = s_np;
-    const int G = a.Hq / a.Hkv;
-    const int n0 = a.node_off[b];
-    const int N = a.node_off[b + 1] - n0;
-    const int kvh = seg / ri.mt, mtile = seg - kvh * ri.mt;
-    const int rows = min(kBM, N * G - mtile * kBM);
     const int D = a.D;
-    const bool fast = np <= kFastPieces;
-    // phase 1: per-row maximum, normaliser and (fast path) weights
-    for (int r = threadIdx.x; r < rows; r += kCombThreads) {
-        float M = -INFINITY;
-        for (int p = 0; p < np; ++p) M = fmaxf(M, a.part_m[(long long)s_slot[p] * kBM + r]);
-        float L = 0.f;
-        for (int p = 0; p < np; ++p) {
-            const long long prow = (long long)s_slot[p] * kBM + r;
-            const float m = a.part_m[prow];
-            const float w = m == -INFINITY ? 0.f : __expf(m - M);
-            L += w * a.part_l[prow];
-            if (fast) s_w[p][r] = w;
+
+    // phase 1: per-row M and 1 / L
+    {
+        const int r = threadIdx.x & (kCombRows - 1), j = threadIdx.x / kCombRows;
+        float fm = -INFINITY, fl = 0.f;
+        if (r < rows) {
+            for (int p = j; p < np; p += kCombFold) {
+                const long long prow = (long long)s_slot[p] * kBM + r0 + r;
+                const float m = a.part_m[prow], l = a.part_l[prow];
+                if (m == -INFINITY) continue;
+                if (m > fm) {
+                    fl = fl * __expf(fm - m) + l;  // fm = -inf: fl = 0
+                    fm = m;
+                } else {
+                    fl += l * __expf(m - fm);
+                }
+            }
         }
-        s_M[r] = M;
-        s_L[r] = L;
-        if (fast)
-            for (int p = 0; p < np; ++p) s_w[p][r] /= L;
+        s_fm[j][r] = fm;
+        s_fl[j][r] = fl;
+        __syncthreads();
+        if (threadIdx.x < kCombRows) {
+            float M = -INFINITY;
+#pragma unroll
+            for (int q = 0; q < kCombFold; ++q) M = fmaxf(M, s_fm[q][r]);
+            float L = 0.f;
+#pragma unroll
+            for (int q = 0; q < kCombFold; ++q)
+                if (s_fm[q][r] != -INFINITY) L += s_fl[q][r] * __expf(s_fm[q][r] - M);
+            s_M[r] = M;
+            s_iL[r] = L > 0.f ? 1.f / L : 0.f;
+            if (r < rows) {
+                const int rr = mtile * kBM + r0 + r;
+                const int i = rr / G, h = kvh * G + (rr - i * G);
+                a.lse[(long long)(n0 + i) * a.Hq + h] = M + __logf(L);
+            }
+        }
+        __syncthreads();
     }
-    __syncthreads();
-    // phase 2: outputs, four columns per item; each thread keeps kItems items
-    // in flight so the partial loads of different items overlap
-    constexpr int kItems = kBM * 32 / kCombThreads;  // 16: all (row, column quad) items of D = 128
+
+    // phase 2: the weighted sum of the partial outputs
+    constexpr int kMaxItems = kCombRows * 128 / 4 / kCombThreads;  // 4 for D = 128
     const int d4 = D / 4;
     const int nitems = rows * d4;
-    float4 acc[kItems];
+    float4 acc[kMaxItems];
+    int irow[kMaxItems];
 #pragma unroll
-    for (int k = 0; k < kItems; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int p = 0; p < np; ++p) {
-        const long long base = (long long)s_slot[p] * kBM;
+    for (int k = 0; k < kMaxItems; ++k) {
+        acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        const int x = threadIdx.x + k * kCombThreads;
+        irow[k] = x < nitems ? x / d4 : -1;
+    }
+    for (int p0 = 0; p0 < np; p0 += kCombBatch) {
+        float m[kCombBatch][kMaxItems];
+        float4 o[kCombBatch][kMaxItems];
 #pragma unroll
-        for (int k = 0; k < kItems; ++k) {
-            const int x = threadIdx.x + k * kCombThreads;
-            if (x >= nitems) continue;
-            const int r = x / d4, q = x - r * d4;
-            float w;
-            if (fast) {
-                w = s_w[p][r];
-            } else {
-                const float m = a.part_m[base + r];
-                w = m == -INFINITY ? 0.f : __expf(m - s_M[r]) / s_L[r];
+        for (int q = 0; q < kCombBatch; ++q) {
+            const long long base = p0 + q < np ? (long long)s_slot[p0 + q] * kBM + r0 : -1;
+#pragma unroll
+            for (int k = 0; k < kMaxItems; ++k) {
+                m[q][k] = -INFINITY;
+                o[q][k] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (base >= 0 && irow[k] >= 0) {
+                    const int x = threadIdx.x + k * kCombThreads;
+                    const int r = irow[k], cq = x - r * d4;
+                    m[q][k] = a.part_m[base + r];
+                    o[q][k] = *reinterpret_cast<const float4 *>(a.part_o + (base + r) * D + cq * 4);
+                }
             }
-            const float4 o = *reinterpret_cast<const float4 *>(a.part_o + (base + r) * D + q * 4);
-            acc[k].x += w * o.x;
-            acc[k].y += w * o.y;
-            acc[k].z += w * o.z;
-            acc[k].w += w * o.w;
+        }
+#pragma unroll
+        for (int q = 0; q < kCombBatch; ++q) {
+#pragma unroll
+            for (int k = 0; k < kMaxItems; ++k) {
+                if (irow[k] < 0 || m[q][k] == -INFINITY) continue;
+                const float w = __expf(m[q][k] - s_M[irow[k]]);
+                acc[k].x = fmaf(w, o[q][k].x, acc[k].x);
+                acc[k].y = fmaf(w, o[q][k].y, acc[k].y);
+                acc[k].z = fmaf(w, o[q][k].z, acc[k].z);
+                acc[k].w = fmaf(w, o[q][k].w, acc[k].w);
+            }
         }
     }
 #pragma unroll
-    for (int k = 0; k < kItems; ++k) {
+    for (int k = 0; k < kMaxItems; ++k) {
+        if (irow[k] < 0) continue;
         const int x = threadIdx.x + k * kCombThreads;
-        if (x >= nitems) continue;
-        const int r = x / d4, q = x - r * d4;
-        const int rr = mtile * kBM + r;
+        const int r = irow[k], cq = x - r * d4;
+        const int rr = mtile * kBM + r0 + r;
         const int i = rr / G, h = kvh * G + (rr - i * G);
         const long long orow = (long long)(n0 + i) * a.Hq + h;
-        *reinterpret_cast<float4 *>(a.out + orow * D + q * 4) = acc[k];
-        if (q == 0) a.lse[orow] = s_M[r] + __logf(s_L[r]);
+        const float f = s_iL[r];
+        *reinterpret_cast<float4 *>(a.out + orow * D + cq * 4) =
+            make_float4(acc[k].x * f, acc[k].y * f, acc[k].z * f, acc[k].w * f);
     }
 }
 
@@ -322,7 +368,7 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     else
         attn_tc_kernel<64><<<Gc, kAttnThreads, smem, st>>>(a, info, tmk, tmv);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/main");
-    attn_combine<<<Gc, kCombThreads, (size_t)(B + 1) * sizeof(int), st>>>(a, info);
+    attn_combine<<<dim3(Gc, kCombGroups), kCombThreads, (size_t)(B + 1) * sizeof(int), st>>>(a, info);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/combine");
     return RS_OK;
 }

@@ -145,72 +145,105 @@ entropy_merge(const Ent3 *__restrict__ part, int nchunks, int R, float *__restri
     if (lane == 0) entropy[r] = t.s > 0.f ? (__logf(t.s) - t.w / t.s) : 0.f;
 }
 
-// Per request: push the committed rows' entropies into the history (row
-// order), then Algorithm 1 step 1 in fp64 (k upward, strict '<').
+// Per request: the committed rows' entropies, in row order, extend the
+// history and the newest l entries are kept; a block scan gives every
+// committed row its rank, so each surviving entry is written by its own
+// thread.  Then Algorithm 1 step 1 in fp64 with one lane per k (H_k, C_k)
+// and a warp argmin that keeps the smallest k among equal C_k (the first
+// strict minimum of the upward scan).
 constexpr int kPushThreads = 256;
-constexpr int kPushRows = 1024;  // rows staged in shared memory per pass
+constexpr int kPushWarps = kPushThreads / 32;
+
+// Exclusive prefix of one int per thread over the block (and the block sum).
+__device__ __forceinline__ int push_scan(int v, int *s_w, int *total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) s_w[warp] = x;
+    __syncthreads();
+    int before = 0, sum = 0;
+#pragma unroll
+    for (int w = 0; w < kPushWarps; ++w) {
+        const int y = s_w[w];
+        before += w < warp ? y : 0;
+        sum += y;
+    }
+    __syncthreads();  // s_w reusable
+    *total = sum;
+    return before + x - v;
+}
 
 __global__ void __launch_bounds__(kPushThreads)
 gate_push(const float *__restrict__ entropy, const int32_t *__restrict__ row_off,
           const uint8_t *__restrict__ row_commit, rs_params p, float *__restrict__ hist,
           int32_t *__restrict__ hist_n, int32_t *__restrict__ k_star, float *__restrict__ h_best,
           uint8_t *__restrict__ entropy_ok) {
-    const int b = blockIdx.x;
+    const int b = blockIdx.x, tid = threadIdx.x;
     const int r0 = row_off[b], r1 = row_off[b + 1];
-    __shared__ float s_ent[kPushRows];
-    __shared__ uint8_t s_com[kPushRows];
-    __shared__ float s_h[RS_MAX_L];
-    __shared__ int s_n;
     const int l = p.l;
-    if (threadIdx.x == 0) {
-        int n = hist_n[b];
-        n = n < 0 ? 0 : (n > l ? l : n);
-        s_n = n;
-        for (int i = 0; i < l; ++i) s_h[i] = hist[(long long)b * l + i];
-    }
-    for (int base = r0; base < r1; base += kPushRows) {
-        const int rows = min(kPushRows, r1 - base);
-        __syncthreads();  // the previous pass is consumed
-        for (int lr = threadIdx.x; lr < rows; lr += kPushThreads) {
-            s_com[lr] = row_commit[base + lr];
-            s_ent[lr] = entropy[base + lr];
-        }
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            int n = s_n;
-            for (int lr = 0; lr < rows; ++lr) {
-                if (!s_com[lr]) continue;
-                if (n == l) {
-                    for (int i = 1; i < l; ++i) s_h[i - 1] = s_h[i];
-                    s_h[l - 1] = s_ent[lr];
-                } else {
-                    s_h[n++] = s_ent[lr];
-                }
-            }
-            s_n = n;
-        }
-    }
-    if (threadIdx.x != 0) return;
-    const int n = s_n;
-    for (int i = 0; i < l; ++i) hist[(long long)b * l + i] = s_h[i];
-    hist_n[b] = n;
+    __shared__ float s_h[RS_MAX_L];
+    __shared__ int s_w[kPushWarps];
+    int n = hist_n[b];
+    n = n < 0 ? 0 : (n > l ? l : n);
 
-    double c_min = INFINITY, best = INFINITY;
-    int kbest = 0;
-    for (int k = 1; k <= n; ++k) {
-        double s = 0.0;
-        for (int i = n - k; i < n; ++i) s = __dadd_rn(s, (double)s_h[i]);
-        double hk = __ddiv_rn(s, (double)k);
-        double ck = __dadd_rn(hk, __ddiv_rn((double)p.lambda_e, (double)k));
-        if (ck < c_min) {
-            c_min = ck;
-            best = hk;
-            kbest = k;
+    // committed rows c; the newest m = min(c, l) of them and the newest
+    // keep = min(n, l - m) old entries form the new history
+    int cnt = 0;
+    for (int r = r0 + tid; r < r1; r += kPushThreads) cnt += row_commit[r] != 0;
+    int c = 0;
+    (void)push_scan(cnt, s_w, &c);
+    const int m = c < l ? c : l;
+    const int keep = n < l - m ? n : l - m;
+    const int nn = keep + m;
+    const float old = tid < keep ? hist[(long long)b * l + n - keep + tid] : 0.f;
+    if (tid < keep) s_h[tid] = old;
+    int carry = 0;
+    for (int base = r0; base < r1; base += kPushThreads) {
+        const int r = base + tid;
+        const bool f = r < r1 && row_commit[r] != 0;
+        int tot = 0;
+        const int q = carry + push_scan(f ? 1 : 0, s_w, &tot);
+        if (f && q >= c - m) s_h[keep + q - (c - m)] = entropy[r];
+        carry += tot;
+    }
+    __syncthreads();
+    if (tid < nn) hist[(long long)b * l + tid] = s_h[tid];
+    if (tid >= 32) return;
+
+    const int k = tid + 1;
+    double ck = INFINITY, hk = INFINITY;
+    if (k <= nn) {
+        double sum = 0.0;
+        for (int i = nn - k; i < nn; ++i) sum = __dadd_rn(sum, (double)s_h[i]);
+        hk = __ddiv_rn(sum, (double)k);
+        ck = __dadd_rn(hk, __ddiv_rn((double)p.lambda_e, (double)k));
+        if (ck != ck) ck = INFINITY;  // a NaN never wins the strict comparison
+    }
+    int bk = k;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const double oc = __shfl_xor_sync(0xffffffffu, ck, o);
+        const double oh = __shfl_xor_sync(0xffffffffu, hk, o);
+        const int ok = __shfl_xor_sync(0xffffffffu, bk, o);
+        if (oc < ck || (oc == ck && ok < bk)) {
+            ck = oc;
+            hk = oh;
+            bk = ok;
         }
     }
-    k_star[b] = kbest;
-    h_best[b] = (float)best;
-    entropy_ok[b] = (uint8_t)(kbest > 0 && best <= (double)p.theta_entropy);
+    if (tid == 0) {
+        hist_n[b] = nn;
+        const bool found = ck < INFINITY;
+        const int kbest = found ? bk : 0;
+        const double best = found ? hk : INFINITY;
+        k_star[b] = kbest;
+        h_best[b] = (float)best;
+        entropy_ok[b] = (uint8_t)(kbest > 0 && best <= (double)p.theta_entropy);
+    }
 }
 
 // The three launches of a gate call over the chunk triples in `part`.
