@@ -77,18 +77,37 @@ __device__ __forceinline__ MS ms_shfl(MS a, int o) {
               __shfl_xor_sync(0xffffffffu, a.w, o)};
 }
 
-// Descending bitonic sort of one float per lane across the warp.
-__device__ __forceinline__ float warp_sort_desc(float x, int lane) {
+// Bitonic sort of one float per lane within aligned groups of G lanes (a
+// power of two <= 32), every group ending in descending order: lane g G + i
+// holds the group's (i + 1)-th largest value.
+template <int G>
+__device__ __forceinline__ float group_sort_desc(float x, int lane) {
 #pragma unroll
-    for (int k = 2; k <= 32; k <<= 1) {
+    for (int k = 2; k <= G; k <<= 1) {
 #pragma unroll
         for (int j = k >> 1; j > 0; j >>= 1) {
             const float y = __shfl_xor_sync(0xffffffffu, x, j);
-            const bool keep_max = ((lane & j) == 0) == ((lane & k) == 0);
+            const bool desc = (k == G) || ((lane & k) == 0);
+            const bool keep_max = ((lane & j) == 0) == desc;
             x = keep_max ? fmaxf(x, y) : fminf(x, y);
         }
     }
     return x;
+}
+
+// The warp maximum and the largest over the warp's G-lane groups of the
+// group's beta-th largest lane value (beta <= G).
+template <int G>
+__device__ __forceinline__ void warp_max_and_bound(float mx, int lane, int beta, float *wmax, float *bound) {
+    const float sorted = group_sort_desc<G>(mx, lane);
+    float m = -INFINITY, t = -INFINITY;
+#pragma unroll
+    for (int g = 0; g < 32; g += G) {
+        m = fmaxf(m, __shfl_sync(0xffffffffu, sorted, g));
+        t = fmaxf(t, __shfl_sync(0xffffffffu, sorted, g + beta - 1));
+    }
+    *wmax = m;
+    *bound = t;
 }
 
 // cp.async: per-thread asynchronous global -> shared copies.  A thread's
@@ -106,11 +125,11 @@ __device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_
 // Start copying the logits this thread will hold of work item `item` = (row,
 // chunk) into `stage` (the same slots it later reads; ids >= V are skipped).
 template <bool kVec>
-__device__ __forceinline__ void fetch_item(const float *__restrict__ logits, int V, int nchunks, long long item,
+__device__ __forceinline__ void fetch_item(const float *__restrict__ logits, int V, int nchunks, int item,
                                            float *stage) {
-    const long long r = item / nchunks;
-    const int c0 = (int)(item - r * nchunks) * kAccChunk;
-    const float *row = logits + r * (long long)V;
+    const int r = item / nchunks;
+    const int c0 = (item - r * nchunks) * kAccChunk;
+    const float *row = logits + (long long)r * V;
     const int tid = threadIdx.x;
     if (kVec) {
 #pragma unroll
@@ -165,17 +184,11 @@ struct RowsShared {
 // barrier is needed at the end: a copy is next written two items later, after
 // every thread has passed the first barrier of the item in between.
 template <bool kVec, bool kEnt>
-__device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int nchunks, int beta, long long blk,
+__device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int c0, int beta, int blk,
                                           VI *__restrict__ cand, MS *__restrict__ part, RowsShared &sh, int rw) {
-    const int c0 = (int)(blk % nchunks) * kAccChunk;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     constexpr float kL2E = 1.4426950408889634f;
-    MS *sms = sh.sms;
-    float *s_thr = sh.thr;
-    auto &s_wtop = sh.wtop;
-    VI *s_cbuf = sh.cbuf;
-    int &s_cnt = sh.cnt;
-    if (tid == 0) s_cnt = 0;
+    if (tid == 0) sh.cnt = 0;
 
     // logit id of register j (padding slots have ids >= V)
     auto id_of = [&](int j) -> int {
@@ -183,34 +196,33 @@ __device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int 
         return c0 + j * kAccThreads + tid;
     };
 
-    // lane maximum (pairwise), then the warp maximum from the sorted lane
-    // maxima (the sort also gives the top-beta threshold below); every lane
-    // exponentiates against the warp maximum, so the warp's (max, sum e, sum
-    // e (z - max)) triple is a plain warp sum.
+    // lane maximum; the warp maximum and a lower bound on the chunk's beta-th
+    // largest logit from the sorted lane maxima: the warp holds beta lane
+    // maxima >= its beta-th largest, and each is a logit of the chunk.  Every lane exponentiates against the warp
+    // maximum, so the warp's (max, sum e, sum e (z - max)) is a plain sum.
     float m8[8];
 #pragma unroll
     for (int q = 0; q < 8; ++q) m8[q] = fmaxf(fmaxf(v[q], v[q + 8]), fmaxf(v[q + 16], v[q + 24]));
     const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
                            fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
-    const float sorted = warp_sort_desc(mx, lane);
-    const float wmax = __shfl_sync(0xffffffffu, sorted, 0);
-    const float thr_w = __shfl_sync(0xffffffffu, sorted, beta - 1);
+    float wmax, thr_w;
+    warp_max_and_bound<32>(mx, lane, beta, &wmax, &thr_w);
     MS t{wmax, 0.f, 0.f};
     if (wmax != -INFINITY) {
+        // base 2: u = (z - max) log2(e), e = 2^u; sum e (z - max) = ln 2 sum e u
+        const float nb = -wmax * kL2E;
         float s4[4] = {0.f, 0.f, 0.f, 0.f};
         float w4[4] = {0.f, 0.f, 0.f, 0.f};
-        if (kEnt) {  // also sum e (z - m) for the row entropy
 #pragma unroll
-            for (int j = 0; j < kAccVpt; ++j) {
-                const float d = fmaxf(v[j] - wmax, -1e30f);  // -inf -> -1e30: e = 0, e*d = 0
-                const float e = sm100::ex2(d * kL2E);
+        for (int j = 0; j < kAccVpt; ++j) {
+            if (kEnt) {
+                const float u = fmaxf(fmaf(v[j], kL2E, nb), -1e30f);  // -inf -> -1e30: e = 0, e u = 0
+                const float e = sm100::ex2(u);
                 s4[j & 3] += e;
-                w4[j & 3] = fmaf(e, d, w4[j & 3]);
+                w4[j & 3] = fmaf(e, u, w4[j & 3]);
+            } else {
+                s4[j & 3] += sm100::ex2(fmaf(v[j], kL2E, nb));
             }
-        } else {
-            const float nb = -wmax * kL2E;
-#pragma unroll
-            for (int j = 0; j < kAccVpt; ++j) s4[j & 3] += sm100::ex2(fmaf(v[j], kL2E, nb));
         }
         float ss = (s4[0] + s4[1]) + (s4[2] + s4[3]);
         float ww = (w4[0] + w4[1]) + (w4[2] + w4[3]);
@@ -220,47 +232,50 @@ __device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int 
             if (kEnt) ww += __shfl_xor_sync(0xffffffffu, ww, o);
         }
         t.s = ss;
-        t.w = ww;
+        t.w = ww * 0.6931471805599453f;
     }
-    if (lane == 0) sms[warp] = t;
+    if (lane == 0) {
+        sh.sms[warp] = t;
+        sh.thr[warp] = thr_w;
+    }
 
     // ---- the chunk's best beta, exactly, in (logit desc, id asc) order ----
-    // A warp's beta-th largest lane maximum T_w is a lower bound on that
-    // warp's beta-th largest logit, hence on the chunk's beta-th largest
-    // logit; so is T = max_w T_w.  Only logits >= T can be in the chunk's
-    // best beta: they are appended to one shared buffer and ranked by warp 0.
-    // If ties overflow the buffer, every warp ranks its own logits and warp 0
+    // Only logits >= T = max over warps of the bounds can be in the chunk's
+    // best beta; they are appended to one shared buffer and ranked by one
+    // warp (each candidate's rank = the number of candidates before it).  If
+    // ties overflow the buffer, every warp ranks its own logits and that warp
     // merges the eight lists instead.
-    if (lane == 0) s_thr[warp] = thr_w;
     __syncthreads();
-    float thr = s_thr[0];
+    float thr = sh.thr[0];
 #pragma unroll
-    for (int w = 1; w < kAccThreads / 32; ++w) thr = fmaxf(thr, s_thr[w]);
+    for (int w = 1; w < kAccThreads / 32; ++w) thr = fmaxf(thr, sh.thr[w]);
+    if (mx >= thr) {
 #pragma unroll
-    for (int j = 0; j < kAccVpt; ++j) {
-        if (v[j] >= thr) {
-            const int id = id_of(j);
-            if (id < V) {
-                const int p = atomicAdd(&s_cnt, 1);
-                if (p < kCandCap) s_cbuf[p] = VI{v[j], id};
+        for (int j = 0; j < kAccVpt; ++j) {
+            if (v[j] >= thr) {
+                const int id = id_of(j);
+                if (id < V) {
+                    const int p = atomicAdd(&sh.cnt, 1);
+                    if (p < kCandCap) sh.cbuf[p] = VI{v[j], id};
+                }
             }
         }
     }
     __syncthreads();
-    const int total = s_cnt;
+    const int total = sh.cnt;
     if (total <= kCandCap) {
         if (warp == rw) {
-            VI prev{INFINITY, -1};
-            for (int k = 0; k < beta; ++k) {
-                VI best{-INFINITY, kNoId};
-                for (int q = lane; q < total; q += 32) {
-                    const VI x = s_cbuf[q];
-                    if (vi_before(prev.v, prev.i, x.v, x.i) && vi_before(x.v, x.i, best.v, best.i)) best = x;
-                }
-                best = warp_vi_best(best);
-                prev = best;
-                if (lane == 0) cand[blk * beta + k] = best;
+            VI x0 = lane < total ? sh.cbuf[lane] : VI{-INFINITY, kNoId};
+            VI x1 = lane + 32 < total ? sh.cbuf[lane + 32] : VI{-INFINITY, kNoId};
+            int r0 = 0, r1 = 0;
+            for (int q = 0; q < total; ++q) {
+                const VI y = sh.cbuf[q];
+                r0 += vi_before(y.v, y.i, x0.v, x0.i);
+                r1 += vi_before(y.v, y.i, x1.v, x1.i);
             }
+            if (lane < total && r0 < beta) cand[(long long)blk * beta + r0] = x0;
+            if (lane + 32 < total && r1 < beta) cand[(long long)blk * beta + r1] = x1;
+            if (lane >= total && lane < beta) cand[(long long)blk * beta + lane] = VI{-INFINITY, kNoId};
         }
     } else {
         VI prev{INFINITY, -1};
@@ -274,7 +289,7 @@ __device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int 
             }
             best = warp_vi_best(best);
             prev = best;
-            if (lane == 0) s_wtop[warp][k] = best;
+            if (lane == 0) sh.wtop[warp][k] = best;
         }
         __syncthreads();
         if (warp == rw) {
@@ -283,21 +298,22 @@ __device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int 
             for (int k = 0; k < beta; ++k) {
                 VI best{-INFINITY, kNoId};
                 for (int q = lane; q < kW * beta; q += 32) {
-                    const VI x = s_wtop[q / beta][q % beta];
+                    const VI x = sh.wtop[q / beta][q % beta];
                     if (x.i != kNoId && vi_before(prevb.v, prevb.i, x.v, x.i) &&
                         vi_before(x.v, x.i, best.v, best.i))
                         best = x;
                 }
                 best = warp_vi_best(best);
                 prevb = best;
-                if (lane == 0) cand[blk * beta + k] = best;
+                if (lane == 0) cand[(long long)blk * beta + k] = best;
             }
         }
     }
-    if (warp == rw && lane == 0) {
-        MS a = sms[0];
-        for (int w = 1; w < kAccThreads / 32; ++w) a = ms_merge(a, sms[w]);
-        part[blk] = a;
+    if (warp == rw) {  // the eight warp triples, merged as a 3-level tree
+        MS a = lane < kAccThreads / 32 ? sh.sms[lane] : MS{-INFINITY, 0.f, 0.f};
+#pragma unroll
+        for (int o = 4; o > 0; o >>= 1) a = ms_merge(a, ms_shfl(a, o));
+        if (lane == 0) part[blk] = a;
     }
 }
 
@@ -308,23 +324,24 @@ constexpr size_t kRowsSmem = (size_t)kRowsStages * kAccChunk * sizeof(float);
 
 template <bool kVec, bool kEnt>
 __global__ void __launch_bounds__(kAccThreads, 3)
-accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, long long n_items,
+accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, int n_items,
             VI *__restrict__ cand, MS *__restrict__ part) {
     __shared__ RowsShared sh[2];
     extern __shared__ __align__(16) float s_stage[];  // kRowsStages x kAccChunk
-    const long long step = gridDim.x;
-    long long item = blockIdx.x;
+    const int step = gridDim.x;
+    int item = blockIdx.x;
     if (item < n_items) fetch_item<kVec>(logits, V, nchunks, item, s_stage);
     cp_async_commit();
     for (int k = 0; item < n_items; ++k, item += step) {
         float *cur = s_stage + (k & 1) * kAccChunk;
         float *nxt = s_stage + ((k + 1) & 1) * kAccChunk;
-        if (item + step < n_items) fetch_item<kVec>(logits, V, nchunks, item + step, nxt);
+        if (item < n_items - step) fetch_item<kVec>(logits, V, nchunks, item + step, nxt);
         cp_async_commit();
         cp_async_wait_1();  // this thread's copies of `item` have landed
+        const int c0 = (item % nchunks) * kAccChunk;
         float v[kAccVpt];
-        read_item<kVec>(cur, V, (int)(item % nchunks) * kAccChunk, v);
-        rows_item<kVec, kEnt>(v, V, nchunks, beta, item, cand, part, sh[k & 1], k % (kAccThreads / 32));
+        read_item<kVec>(cur, V, c0, v);
+        rows_item<kVec, kEnt>(v, V, c0, beta, item, cand, part, sh[k & 1], k % (kAccThreads / 32));
     }
 }
 
@@ -709,7 +726,8 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
     float *rowmax = cv.take<float>((size_t)R);
     if (R > 0) {
         const long long blocks = (long long)R * nchunks;
-        RS_CHECK_ARG(blocks < (1ll << 31), "rs_accept: R*chunks too large");
+        RS_CHECK_ARG(blocks < (1ll << 30), "rs_accept: R*chunks too large");
+        const int n_items = (int)blocks;
         const bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
         const bool ent = entropy != nullptr;
         const unsigned grid = (unsigned)std::min<long long>(blocks, 3ll * num_sms());
@@ -734,13 +752,13 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
             attr_done[dev] = 1;
         }
         if (vec && ent)
-            accept_rows<true, true><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, blocks, cand, part);
+            accept_rows<true, true><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, n_items, cand, part);
         else if (vec)
-            accept_rows<true, false><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, blocks, cand, part);
+            accept_rows<true, false><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, n_items, cand, part);
         else if (ent)
-            accept_rows<false, true><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, blocks, cand, part);
+            accept_rows<false, true><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, n_items, cand, part);
         else
-            accept_rows<false, false><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, blocks, cand, part);
+            accept_rows<false, false><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, n_items, cand, part);
         RS_CHECK_LAUNCH("rs_accept/accept_rows");
         accept_merge<<<(R + kMergeThreads / 32 - 1) / (kMergeThreads / 32), kMergeThreads, 0, st>>>(
             cand, part, nchunks, p.beta, R, argmax, topk, lse, entropy, rowmax);
@@ -748,8 +766,8 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
     }
     if (B > 0) {
         accept_decide<<<B, kDecThreads, 0, st>>>(logits, V, node_off, tokens, parents, source, chain, sel_pos,
-                                                 tok_off, p, acc_cap, argmax, topk, lse, rowmax, p_tok, acc_len, acc_nodes,
-                                                 bonus, winner, commit, scores, status);
+                                                 tok_off, p, acc_cap, argmax, topk, lse, rowmax, p_tok, acc_len,
+                                                 acc_nodes, bonus, winner, commit, scores, status);
         RS_CHECK_LAUNCH("rs_accept/accept_decide");
     }
     return RS_OK;
