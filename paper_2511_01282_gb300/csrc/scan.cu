@@ -1,19 +1,27 @@
 // scan.cu -- rs_match_scan: retrieval and feedback-driven candidate
 // selection (Section 3.3 "Selection Algorithm"; Algorithm 1 l.9-11).
 //
-// One cluster of 8 CTAs (256 threads each) per request; CTA c scans the c-th
-// eighth of the candidate positions [k-1, t-2].  Per window of 8192
-// positions, warp w, step j tests positions 32 (w + 8 j) + lane against the
-// key (both staged in shared memory) and its ballot is one 32-bit word of
-// the window's match bitmask; thread i owns word i.  Pass 1 counts the slice's
-// matches and keeps each thread's best top_c matches (score desc, position
-// desc) in a small register list, merged per CTA.  After a cluster barrier
-// every CTA reads its peers' counts through distributed shared memory, so
-// pass 2 writes its positions at their global ascending rank (a block scan
-// of word popcounts orders them within a window) -- no sort.  CTA 0 merges
-// the eight per-CTA top_c lists and gathers the selected continuations.  The
-// cluster's CTAs are co-scheduled and all of them pass the same two cluster
-// barriers, so nothing waits on a CTA that is not running.
+// One cluster of 8 CTAs (256 threads each) per request.  A buffer whose
+// candidate positions [0, t-2] fit one window of 8192 is handled by CTA 0
+// alone (the other seven leave at once and no cluster barrier is used);
+// otherwise CTA c scans the c-th eighth of the positions.  A window is staged
+// in shared memory in one round of loads issued together: its tokens with
+// the k-1 before it, its scores, and the key.  Warp w, step j tests positions
+// 32 (w + 8 j) + lane against the key; the ballot is one 32-bit word of the
+// window's match bitmask, and thread i owns word i.  One block scan of the
+// word popcounts gives the CTA's match count and every thread's rank, so
+// positions are written at their global ascending rank with no sort.
+// Matches whose score clears theta_score are appended to a shared buffer and
+// each is ranked by counting the buffered matches before it in (score desc,
+// position desc) order, which gives the CTA's best top_c in one pass; if more
+// match than the buffer holds, per-thread lists merged block-wide are used
+// instead.  In the split case every CTA pushes its count
+// to all peers and its best top_c to CTA 0 through distributed shared memory
+// before one cluster barrier; after it nobody touches another CTA's shared
+// memory.  CTA 0 ranks the (at most 64) listed matches the same way and
+// gathers the selected continuations (from the staged window when it alone
+// scanned the buffer).  A slice that
+// spans several windows stages them in turn, and again for the position pass.
 #include <cooperative_groups.h>
 #include <math.h>
 
@@ -28,6 +36,8 @@ constexpr int kScanCluster = 8;
 constexpr int kScanThreads = 256;
 constexpr int kScanWarps = kScanThreads / 32;
 constexpr int kWin = kScanThreads * 32;  // positions per window
+constexpr int kHalo = RS_MAX_L - 1;      // tokens staged before the window
+constexpr int kScanCand = 256;           // matches ranked from the shared buffer
 
 // (s, p) before (s2, p2): higher score first, then the more recent position
 __device__ __forceinline__ bool sp_before(float s, int p, float s2, int p2) {
@@ -35,14 +45,21 @@ __device__ __forceinline__ bool sp_before(float s, int p, float s2, int p2) {
 }
 
 struct ScanShared {
-    int tok[kWin + RS_MAX_L];       // buffer tokens [w0 - (k - 1), w0 + kWin) of the current window
+    int tok[kHalo + kWin];   // X[w0 - kHalo, w0 + kWin) (unwritten outside [0, t))
+    float sc[kWin];          // S[w0, w0 + kWin)
     uint32_t bits[kWin / 32];
+    float cs[kScanCand];     // matches with S >= theta_score (first kScanCand)
+    int cp[kScanCand];
+    int ccnt;
     int warp_sums[kScanWarps + 1];
     float wv[kScanWarps];
     int wp[kScanWarps];
     int key[RS_MAX_L];
-    long long cnt;                  // this CTA's match count (read by the peers)
-    float top_s[RS_MAX_TOPC];       // this CTA's best top_c (read by CTA 0)
+    long long peer_cnt[kScanCluster];           // match count of each CTA (pushed by its owner)
+    float peer_s[kScanCluster][RS_MAX_TOPC];    // CTA 0: each CTA's best top_c
+    int peer_p[kScanCluster][RS_MAX_TOPC];
+    int peer_n[kScanCluster];
+    float top_s[RS_MAX_TOPC];                   // this CTA's best top_c
     int top_p[RS_MAX_TOPC];
     int ntop;
     int sel[RS_MAX_TOPC];
@@ -59,47 +76,87 @@ __device__ __forceinline__ int block_excl_scan(int v, ScanShared &sh, int *total
     }
     if (lane == 31) sh.warp_sums[warp] = x;
     __syncthreads();
-    if (warp == 0) {
-        const int w = lane < kScanWarps ? sh.warp_sums[lane] : 0;
-        int z = w;
+    int before = 0, sum = 0;
 #pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, z, o);
-            if (lane >= o) z += y;
-        }
-        if (lane < kScanWarps) sh.warp_sums[lane] = z - w;
-        if (lane == kScanWarps - 1) sh.warp_sums[kScanWarps] = z;
+    for (int w = 0; w < kScanWarps; ++w) {
+        const int y = sh.warp_sums[w];
+        before += w < warp ? y : 0;
+        sum += y;
     }
-    __syncthreads();
-    const int r = sh.warp_sums[warp] + x - v;
-    *total = sh.warp_sums[kScanWarps];
     __syncthreads();  // warp_sums reusable
-    return r;
+    *total = sum;
+    return before + x - v;
 }
 
-// The match bitmask of window [w0, w0 + kWin) restricted to [lo, hi).  The
-// window's tokens (and the k - 1 before it) are first staged in shared
-// memory with independent coalesced loads.
-__device__ __forceinline__ void window_bits(const int32_t *__restrict__ X, long long t, int k, long long w0,
-                                            long long lo, long long hi, ScanShared &sh) {
+// Stage window [w0, w0 + kWin): tokens from w0 - kHalo that lie in
+// [0, tok_hi), scores of the positions below `hi`, as asynchronous 4-byte
+// copies (all in flight at once; the caller waits and synchronises).  Slots
+// outside those ranges are left unwritten: the key test reads only tokens of
+// candidate positions p - i, 0 <= p - i < hi, and a gathered span only
+// tokens below t.
+__device__ __forceinline__ void cp_async4(void *smem, const void *gmem) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(smem))),
+                 "l"(gmem)
+                 : "memory");
+}
+
+__device__ __forceinline__ void stage_window(const int32_t *__restrict__ X, const float *__restrict__ S,
+                                             long long tok_hi, long long hi, long long w0, ScanShared &sh) {
+    const long long a = w0 - kHalo;
+    const int j0 = (int)(a < 0 ? -a : 0);
+    const int j1 = (int)(tok_hi - a < kHalo + kWin ? tok_hi - a : kHalo + kWin);
+    for (int j = j0 + threadIdx.x; j < j1; j += kScanThreads) cp_async4(&sh.tok[j], X + a + j);
+    const int n = (int)(hi - w0 < kWin ? hi - w0 : kWin);
+    for (int j = threadIdx.x; j < n; j += kScanThreads) cp_async4(&sh.sc[j], S + w0 + j);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+__device__ __forceinline__ void stage_wait() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
+// The match bitmask of the staged window restricted to [lo, hi).  The key is
+// in registers (key[i] = X[t - k + i]).  Thread (warp, lane) tests positions
+// w0 + 256 j + 32 warp + lane, j = 0..31.  Pass 1 has no branches: one
+// shared load and compare of the last token per position and a ballot per
+// word, kept by lane j.  Pass 2 visits only the words with a hit and
+// compares the other k - 1 tokens.  The bitmask is written with one store per
+// thread.
+__device__ __forceinline__ void window_bits(const int (&key)[RS_MAX_L], int k, long long w0, long long lo,
+                                            long long hi, ScanShared &sh) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const long long t_lo = w0 - (k - 1);
-    for (int j = threadIdx.x; j < kWin + k - 1; j += kScanThreads) {
-        const long long idx = t_lo + j;
-        sh.tok[j] = (idx >= 0 && idx < t) ? X[idx] : -1;
-    }
-    __syncthreads();
+    const int klast = key[k - 1];
+    const int r0 = warp * 32 + lane;  // offset of this thread's j = 0 position in the window
+    // valid j: lo <= w0 + r0 + 256 j < hi
+    const long long dlo = lo - w0 - r0, dhi = hi - w0 - r0;
+    const int jlo = dlo <= 0 ? 0 : (int)((dlo + kScanThreads - 1) / kScanThreads);
+    const int jhi = dhi <= 0 ? 0 : (int)((dhi + kScanThreads - 1) / kScanThreads);
+    const int *tk = sh.tok + kHalo + r0;
+    uint32_t mine = 0;
 #pragma unroll 8
     for (int j = 0; j < 32; ++j) {
-        const int word = warp + kScanWarps * j;
-        const long long p = w0 + (long long)word * 32 + lane;
-        const int base = word * 32 + lane;  // tokens of p: tok[base .. base + k - 1]
-        bool m = p >= lo && p < hi;
-        for (int i = 0; i < k; ++i) m &= (sh.tok[base + i] == sh.key[i]);
-        const unsigned bal = __ballot_sync(0xffffffffu, m);
-        if (lane == 0) sh.bits[word] = bal;
+        const bool m = (j >= jlo) & (j < jhi) & (tk[j * kScanThreads] == klast);
+        const uint32_t bal = __ballot_sync(0xffffffffu, m);
+        mine = lane == j ? bal : mine;
     }
-    __syncthreads();
+    if (k > 1) {
+        uint32_t words = __ballot_sync(0xffffffffu, mine != 0u);
+        while (words) {
+            const int j = __ffs(words) - 1;
+            words &= words - 1;
+            bool m = (j >= jlo) & (j < jhi) & (tk[j * kScanThreads] == klast);
+            for (int i = 1; i < k; ++i) m = m && (tk[j * kScanThreads - i] == key[k - 1 - i]);
+            const uint32_t bal = __ballot_sync(0xffffffffu, m);
+            mine = lane == j ? bal : mine;
+        }
+    }
+    sh.bits[warp + kScanWarps * lane] = mine;
+}
+
+// Rank of (s, p) among n distinct (score, position) pairs in shared memory:
+// the number of pairs before it in (score desc, position desc) order.
+__device__ __forceinline__ int sp_rank(float s, int p, const float *cs, const int *cp, int n) {
+    int r = 0;
+    for (int q = 0; q < n; ++q) r += sp_before(cs[q], cp[q], s, p);
+    return r;
 }
 
 // Best head of the block's register lists; every thread gets it.
@@ -146,12 +203,13 @@ match_scan_kernel(const int32_t *__restrict__ tokens, const int64_t *__restrict_
     const int crank = (int)cluster.block_rank();
     const int b = blockIdx.y;
     const int tid = threadIdx.x;
+    extern __shared__ __align__(16) unsigned char scan_smem[];
+    ScanShared &sh = *reinterpret_cast<ScanShared *>(scan_smem);
     const long long t0 = tok_off[b];
     const long long t = tok_off[b + 1] - t0;
     const int32_t *X = tokens + t0;
     const float *S = scores + t0;
     const int k = k_star[b];
-    __shared__ ScanShared sh;
 
     int st = 0;
     bool run = k > 0 && (gate_ok == nullptr || gate_ok[b] != 0);
@@ -160,21 +218,32 @@ match_scan_kernel(const int32_t *__restrict__ tokens, const int64_t *__restrict_
         run = false;
     }
     if (run && (long long)k > t) run = false;
-    if (run && tid < k) sh.key[tid] = X[t - k + tid];
 
-    // this CTA's slice of the candidate positions [k-1, t-2]
+    // this CTA's slice [lo, hi) of the positions [0, t-2]; matches need p >= k-1
+    // t <= kWin: the tokens [0, t) all fit the staged window (after the halo)
+    const bool solo = !run || t <= kWin;  // CTA 0 alone, no cluster barrier
+    if (solo && crank != 0) return;
     long long lo = 0, hi = 0;
     if (run) {
-        const long long first = k - 1, n = (t - 1) - first;
-        long long per = (n + kScanCluster - 1) / kScanCluster;
+        const long long n = t - 1;
+        long long per = solo ? n : (n + kScanCluster - 1) / kScanCluster;
         per = (per + 31) / 32 * 32;
-        lo = first + (long long)crank * per;
-        hi = lo + per < t - 1 ? lo + per : t - 1;
+        lo = (long long)crank * per;
+        hi = lo + per < n ? lo + per : n;
         if (lo > hi) lo = hi;
     }
+    const long long plo = lo > k - 1 ? lo : (long long)(k - 1);
+    const bool single = hi - lo <= kWin;
+    if (tid == 0) sh.ccnt = 0;
+    if (run && tid < k) sh.key[tid] = X[t - k + tid];
+    if (run && lo < hi) stage_window(X, S, solo ? t : hi, hi, lo, sh);
+    stage_wait();
     __syncthreads();
+    int key[RS_MAX_L];
+#pragma unroll
+    for (int i = 0; i < RS_MAX_L; ++i) key[i] = (run && i < k) ? sh.key[i] : -1;
 
-    // ---- pass 1: count, and each thread's best matches ----
+    // ---- pass 1: match bits, count, candidates ----
     float ls[RS_MAX_TOPC];
     int lp[RS_MAX_TOPC];
 #pragma unroll
@@ -182,87 +251,139 @@ match_scan_kernel(const int32_t *__restrict__ tokens, const int64_t *__restrict_
         ls[i] = -INFINITY;
         lp[i] = -1;
     }
-    long long cnt = 0;
+    int cnt = 0, rank = 0;
     for (long long w0 = lo; w0 < hi; w0 += kWin) {
-        window_bits(X, t, k, w0, lo, hi, sh);
+        if (w0 != lo) {
+            __syncthreads();  // the previous window is consumed
+            stage_window(X, S, hi, hi, w0, sh);
+            stage_wait();
+            __syncthreads();
+        }
+        window_bits(key, k, w0, plo, hi, sh);
+        __syncthreads();
         uint32_t rem = sh.bits[tid];
         cnt += __popc(rem);
         while (rem) {
             const int bit = __ffs(rem) - 1;
             rem &= rem - 1;
-            const long long p = w0 + (long long)tid * 32 + bit;
-            const float s = S[p];
-            if (s >= theta_score && sp_before(s, (int)p, ls[RS_MAX_TOPC - 1], lp[RS_MAX_TOPC - 1])) {
+            const int off = tid * 32 + bit;
+            const float s = sh.sc[off];
+            if (!(s >= theta_score)) continue;
+            const int p = (int)(w0 + off);
+            const int q = atomicAdd(&sh.ccnt, 1);
+            if (q < kScanCand) {
+                sh.cs[q] = s;
+                sh.cp[q] = p;
+            }
+            if (sp_before(s, p, ls[RS_MAX_TOPC - 1], lp[RS_MAX_TOPC - 1])) {
                 float cs = s;
-                int cp = (int)p;
+                int cp = p;
 #pragma unroll
-                for (int q = 0; q < RS_MAX_TOPC; ++q) {
-                    if (sp_before(cs, cp, ls[q], lp[q])) {
-                        const float ts = ls[q];
-                        const int tp = lp[q];
-                        ls[q] = cs;
-                        lp[q] = cp;
+                for (int i = 0; i < RS_MAX_TOPC; ++i) {
+                    if (sp_before(cs, cp, ls[i], lp[i])) {
+                        const float ts = ls[i];
+                        const int tp = lp[i];
+                        ls[i] = cs;
+                        lp[i] = cp;
                         cs = ts;
                         cp = tp;
                     }
                 }
             }
         }
-        __syncthreads();  // bits and tok reusable
     }
-    // the CTA's count and best top_c
-    {
-        int c32 = (int)cnt, total = 0;
-        (void)block_excl_scan(c32, sh, &total);
-        if (tid == 0) sh.cnt = total;
-    }
-    int ntop = 0;
-    for (int c = 0; c < top_c; ++c) {
-        float bv;
-        int bp;
-        block_best(ls[0], lp[0], sh, &bv, &bp);
-        if (bp < 0) break;
-        if (tid == 0) {
-            sh.top_s[c] = bv;
-            sh.top_p[c] = bp;
-        }
-        ntop = c + 1;
-        if (lp[0] == bp) {  // the owner pops its head
-#pragma unroll
-            for (int q = 0; q < RS_MAX_TOPC - 1; ++q) {
-                ls[q] = ls[q + 1];
-                lp[q] = lp[q + 1];
+    // the CTA's count; in a single window also every thread's position rank
+    int cta_total = 0;
+    rank = block_excl_scan(cnt, sh, &cta_total);  // single window: cnt = popc(bits[tid])
+    // the CTA's best top_c: rank every buffered candidate by counting
+    const int ncand = sh.ccnt;
+    if (ncand <= kScanCand) {
+        for (int e = tid; e < ncand; e += kScanThreads) {
+            const float sv = sh.cs[e];
+            const int pv = sh.cp[e];
+            const int r = sp_rank(sv, pv, sh.cs, sh.cp, ncand);
+            if (r < top_c) {
+                sh.top_s[r] = sv;
+                sh.top_p[r] = pv;
             }
-            ls[RS_MAX_TOPC - 1] = -INFINITY;
-            lp[RS_MAX_TOPC - 1] = -1;
         }
+        if (tid == 0) sh.ntop = ncand < top_c ? ncand : top_c;
+    } else {
+        int ntop = 0;
+        for (int c = 0; c < top_c; ++c) {
+            float bv;
+            int bp;
+            block_best(ls[0], lp[0], sh, &bv, &bp);
+            if (bp < 0) break;
+            if (tid == 0) {
+                sh.top_s[c] = bv;
+                sh.top_p[c] = bp;
+            }
+            ntop = c + 1;
+            if (lp[0] == bp) {  // the owner pops its head
+#pragma unroll
+                for (int i = 0; i < RS_MAX_TOPC - 1; ++i) {
+                    ls[i] = ls[i + 1];
+                    lp[i] = lp[i + 1];
+                }
+                ls[RS_MAX_TOPC - 1] = -INFINITY;
+                lp[RS_MAX_TOPC - 1] = -1;
+            }
+        }
+        if (tid == 0) sh.ntop = ntop;
     }
-    if (tid == 0) sh.ntop = ntop;
-    cluster.sync();
 
-    // ---- the slice's global rank; pass 2 writes positions in order ----
-    long long offset = 0, total = 0;
-    for (int r = 0; r < kScanCluster; ++r) {
-        const long long c = *cluster.map_shared_rank(&sh.cnt, r);
-        if (r < crank) offset += c;
-        total += c;
+    // ---- the slice's global rank (pushed counts); positions in ascending order ----
+    long long offset = 0, total = cta_total;
+    if (!solo) {
+        __syncthreads();  // this CTA's top list is complete
+        if (tid < kScanCluster) *cluster.map_shared_rank(&sh.peer_cnt[crank], tid) = cta_total;
+        if (tid < RS_MAX_TOPC) {
+            *cluster.map_shared_rank(&sh.peer_s[crank][tid], 0) = sh.top_s[tid];
+            *cluster.map_shared_rank(&sh.peer_p[crank][tid], 0) = sh.top_p[tid];
+        }
+        if (tid == 0) *cluster.map_shared_rank(&sh.peer_n[crank], 0) = sh.ntop;
+        cluster.sync();  // the only cluster barrier: every push is visible after it
+        total = 0;
+        for (int r = 0; r < kScanCluster; ++r) {
+            const long long c = sh.peer_cnt[r];
+            if (r < crank) offset += c;
+            total += c;
+        }
+    } else {
+        __syncthreads();
     }
     if (run && offset < pos_cap) {
-        long long base = offset;
-        for (long long w0 = lo; w0 < hi && base < pos_cap; w0 += kWin) {
-            window_bits(X, t, k, w0, lo, hi, sh);
-            uint32_t rem = sh.bits[tid];
-            int wtotal = 0;
-            const int rank = block_excl_scan(__popc(rem), sh, &wtotal);
+        if (single) {
+            uint32_t rem = lo < hi ? sh.bits[tid] : 0u;
             int i = 0;
             while (rem) {
                 const int bit = __ffs(rem) - 1;
                 rem &= rem - 1;
-                const long long idx = base + rank + i++;
-                if (idx < pos_cap) pos[(long long)b * pos_cap + idx] = (int32_t)(w0 + (long long)tid * 32 + bit);
+                const long long idx = offset + rank + i++;
+                if (idx < pos_cap) pos[(long long)b * pos_cap + idx] = (int32_t)(lo + (long long)tid * 32 + bit);
             }
-            base += wtotal;
-            __syncthreads();  // bits reusable
+        } else {
+            long long base = offset;
+            for (long long w0 = lo; w0 < hi && base < pos_cap; w0 += kWin) {
+                __syncthreads();  // the previous window is consumed
+                stage_window(X, S, hi, hi, w0, sh);
+                stage_wait();
+                __syncthreads();
+                window_bits(key, k, w0, plo, hi, sh);
+                __syncthreads();
+                uint32_t rem = sh.bits[tid];
+                int wtotal = 0;
+                const int r0 = block_excl_scan(__popc(rem), sh, &wtotal);
+                int i = 0;
+                while (rem) {
+                    const int bit = __ffs(rem) - 1;
+                    rem &= rem - 1;
+                    const long long idx = base + r0 + i++;
+                    if (idx < pos_cap) pos[(long long)b * pos_cap + idx] = (int32_t)(w0 + (long long)tid * 32 + bit);
+                }
+                base += wtotal;
+            }
         }
     }
 
@@ -271,49 +392,32 @@ match_scan_kernel(const int32_t *__restrict__ tokens, const int64_t *__restrict_
         const long long stored = total < pos_cap ? total : pos_cap;
         for (long long i = stored + tid; i < pos_cap; i += kScanThreads) pos[(long long)b * pos_cap + i] = -1;
         if (total > pos_cap) st |= RS_ST_TRUNCATED;
-        if (tid < 32) {
-            // up to kScanCluster * RS_MAX_TOPC = 64 candidates, two per lane
-            float cv[2];
-            int cpos[2];
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int e = tid + 32 * h, r = e / RS_MAX_TOPC, q = e % RS_MAX_TOPC;
-                cv[h] = -INFINITY;
-                cpos[h] = -1;
-                if (q < *cluster.map_shared_rank(&sh.ntop, r)) {
-                    cv[h] = *cluster.map_shared_rank(&sh.top_s[q], r);
-                    cpos[h] = *cluster.map_shared_rank(&sh.top_p[q], r);
-                }
+        // the cluster's candidates (up to kScanCluster * RS_MAX_TOPC), ranked by counting
+        float *ms = sh.cs;  // reused: the CTA's own buffer is no longer needed
+        int *mp = sh.cp;
+        int nm = 0;
+        if (solo) {
+            nm = sh.ntop;
+            for (int q = tid; q < nm; q += kScanThreads) {
+                ms[q] = sh.top_s[q];
+                mp[q] = sh.top_p[q];
             }
-            int nsel = 0;
-            float pv = INFINITY;
-            int pp = 0x7fffffff;
-            for (int c = 0; c < top_c; ++c) {
-                float hv = -INFINITY;
-                int hp = -1;
-#pragma unroll
-                for (int h = 0; h < 2; ++h)
-                    if (cpos[h] >= 0 && sp_before(pv, pp, cv[h], cpos[h]) && sp_before(cv[h], cpos[h], hv, hp)) {
-                        hv = cv[h];
-                        hp = cpos[h];
-                    }
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) {
-                    const float ov = __shfl_xor_sync(0xffffffffu, hv, o);
-                    const int op = __shfl_xor_sync(0xffffffffu, hp, o);
-                    if (sp_before(ov, op, hv, hp)) {
-                        hv = ov;
-                        hp = op;
-                    }
+        } else {
+            for (int r = 0; r < kScanCluster; ++r) {
+                const int n = sh.peer_n[r];
+                if (tid < n) {
+                    ms[nm + tid] = sh.peer_s[r][tid];
+                    mp[nm + tid] = sh.peer_p[r][tid];
                 }
-                if (hp < 0) break;
-                if (tid == 0) sh.sel[c] = hp;
-                nsel = c + 1;
-                pv = hv;
-                pp = hp;
+                nm += n;
             }
-            if (tid == 0) sh.ntop = nsel;  // own copy: the peers have been read
         }
+        __syncthreads();
+        if (tid < nm) {
+            const int r = sp_rank(ms[tid], mp[tid], ms, mp, nm);
+            if (r < top_c) sh.sel[r] = mp[tid];
+        }
+        if (tid == 0) sh.ntop = nm < top_c ? nm : top_c;
         __syncthreads();
         const int nsel = sh.ntop;
         for (int i = tid; i < top_c * span_len; i += kScanThreads) {
@@ -323,7 +427,8 @@ match_scan_kernel(const int32_t *__restrict__ tokens, const int64_t *__restrict_
                 const long long p = sh.sel[c];
                 long long len = t - 1 - p;
                 if (len > span_len) len = span_len;
-                if (j < len) v = X[p + 1 + j];
+                // solo: X[p + 1 + j], p + 1 + j <= t - 1, is staged at tok[kHalo + p + 1 + j]
+                if (j < len) v = solo ? sh.tok[kHalo + p + 1 + j] : __ldg(X + p + 1 + j);
             }
             spans[(long long)b * top_c * span_len + i] = v;
         }
@@ -344,7 +449,6 @@ match_scan_kernel(const int32_t *__restrict__ tokens, const int64_t *__restrict_
             status[b] = st;
         }
     }
-    cluster.sync();  // the peers' shared memory stays valid until CTA 0 is done
 }
 
 }  // namespace
@@ -376,7 +480,19 @@ extern "C" rs_status rs_match_scan(const int32_t *tokens, const int64_t *tok_off
                             n_sel && status && (pos || pos_cap == 0)),
                  "rs_match_scan: null pointer");
     if (B == 0) return RS_OK;
-    match_scan_kernel<<<dim3(kScanCluster, B), kScanThreads, 0, (cudaStream_t)stream>>>(
+    static int attr_done[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(match_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)sizeof(ScanShared));
+        if (e != cudaSuccess) {
+            set_error("rs_match_scan: cudaFuncSetAttribute: %s", cudaGetErrorString(e));
+            return RS_ERR_CUDA;
+        }
+        attr_done[dev] = 1;
+    }
+    match_scan_kernel<<<dim3(kScanCluster, B), kScanThreads, sizeof(ScanShared), (cudaStream_t)stream>>>(
         tokens, tok_off, k_star, gate_ok, scores, p.theta_score, p.top_c, p.span_len, pos_cap, count, pos,
         sel_pos, sel_len, spans, n_sel, status);
     RS_CHECK_LAUNCH("rs_match_scan");

@@ -196,3 +196,43 @@ def test_cuda_graph_replay_matches_eager():
         assert rs.rs_launch_count() == n0  # replays do not go through the host entry points
         for k, v in eager.items():
             assert (host(st.out[k]) == v).all(), (fused, k)
+
+
+def _scan_direct(tokens, tok_off, ks, ok, scores, theta, top_c, span_len, pos_cap):
+    B = len(tok_off) - 1
+    z = lambda *shape: torch.full(shape, -7, dtype=torch.int32, device="cuda")  # noqa: E731
+    out = dict(count=z(B), pos=z(B, pos_cap), sel_pos=z(B, top_c), sel_len=z(B, top_c),
+               spans=z(B, top_c, span_len), n_sel=z(B), status=z(B))
+    p = rs.params(theta_score=theta, top_c=top_c, span_len=span_len)
+    rs.rs_match_scan(_cuda(tokens), _cuda(tok_off), B, _cuda(ks), _cuda(ok), _cuda(scores), p, pos_cap,
+                     out["count"], out["pos"], out["sel_pos"], out["sel_len"], out["spans"], out["n_sel"],
+                     out["status"])
+    torch.cuda.synchronize()
+    return {k: host(v) for k, v in out.items()}
+
+
+@pytest.mark.parametrize("dense", [False, True])
+def test_scan_long_buffers(dense):
+    # buffer lengths at the one-CTA limit (8192), just above it (split over the
+    # cluster, one window per CTA), at the one-window-per-CTA limit (65537) and
+    # well past it (several windows per CTA); dense: a 3-token vocabulary, so
+    # thousands of matches overflow the shared candidate buffer and pos_cap
+    rng = np.random.default_rng(21 + dense)
+    lens = [8192, 8193, 65537, 65538, 150001]
+    V = 3 if dense else 200
+    tok_off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    tokens = rng.integers(0, V, int(tok_off[-1])).astype(np.int32)
+    for b, t in enumerate(lens):  # plant the key earlier so sparse buffers match too
+        a = int(tok_off[b])
+        for q in rng.integers(8, t - 8, 6):
+            tokens[a + q - 3:a + q + 1] = tokens[a + t - 4:a + t]
+    scores = rng.random(int(tok_off[-1])).astype(np.float32)
+    scores[rng.random(scores.size) < 0.1] = 0.75  # ties on the score
+    ks = np.array([1, 2, 3, 4, 2], np.int32)
+    ok = np.ones(len(lens), np.uint8)
+    theta, top_c, span_len, pos_cap = 0.3, 8, 16, 5000
+    got = _scan_direct(tokens, tok_off, ks, ok, scores, theta, top_c, span_len, pos_cap)
+    ref = oracle.match_scan(tokens, tok_off, ks, scores, f32(theta), top_c, span_len, pos_cap, gate_ok=ok)
+    for key in ("count", "pos", "sel_pos", "sel_len", "spans", "n_sel", "status"):
+        assert (got[key] == ref[key]).all(), key
+    assert (ref["n_sel"] > 0).all()
