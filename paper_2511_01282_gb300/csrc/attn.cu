@@ -20,6 +20,8 @@
 #include <cudaTypedefs.h>
 #include <math.h>
 
+#include <algorithm>
+
 #include <mutex>
 
 #include "attn_core.cuh"
@@ -80,62 +82,91 @@ attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_
     if (tid == 0) status[b] = st;
 }
 
-// Block (c, y) merges rows [32 y, 32 y + 32) of the split segment whose first
-// piece is c's last piece (four blocks per segment; the pieces are the
-// partials of the CTAs c .. c1 whose ranges cut the segment).
+// Block (c, y) merges rows [32 y, 32 y + 32) of the split segment CTA c of
+// the attention kernel started (its job record; four blocks per segment).
+// The segment's pieces are the partials of CTA c (slot first_slot) and of
+// slot 0 of every later CTA up to c1 with a non-empty range.
 // Phase 1: thread (row r, lane group j) folds the (m, l) pairs of pieces j,
 // j + 8, ... into a running (max, sum); warp 0 merges the eight folds into the
 // row's M = max_p m_p and 1 / L, L = sum_p e^(m_p - M) l_p.  Phase 2: each
 // thread owns D / 32 (row, 4 head-dim columns) items and sums e^(m_p - M) O_p
-// over the pieces, four pieces per round, so a round keeps 4 x D / 32 float4
-// partial loads and their m_p loads in flight.  The summation order is fixed
-// (piece order), so the result does not depend on timing.
+// over the pieces, two pieces per round, so a round keeps 2 x D / 32 float4
+// partial loads and their m_p loads in flight (the first round is issued
+// before phase 1, so the two phases share one memory round trip).  The
+// summation order is fixed (piece order), so the result does not depend on
+// timing.
 constexpr int kCombThreads = 256;
 constexpr int kCombRows = 32;                    // rows per block
 constexpr int kCombGroups = kBM / kCombRows;     // blocks per split segment
 constexpr int kCombFold = kCombThreads / kCombRows;  // lane groups in phase 1
-constexpr int kCombBatch = 4;                    // pieces per phase-2 round
-constexpr int kMaxPieces = 1024;
+constexpr int kCombBatch = 2;                    // pieces per phase-2 round
 
-__global__ void __launch_bounds__(kCombThreads)
-attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
-    extern __shared__ int s_pref[];
-    __shared__ int s_slot[kMaxPieces];
+__global__ void __launch_bounds__(kCombThreads, 4)  // the 4 x Gc blocks in one wave
+attn_combine(AttnArgs a) {
+    __shared__ int s_slot[kAttnMaxGrid];
     __shared__ float s_fm[kCombFold][kCombRows], s_fl[kCombFold][kCombRows];
     __shared__ float s_M[kCombRows], s_iL[kCombRows];
-    __shared__ int s_np;
-    unit_prefix(info, a.B, s_pref);
-    const long long W = s_pref[a.B];
-    const long long Gc = gridDim.x, c = blockIdx.x;
-    const long long u0 = range_lo(c, W, Gc), u1 = range_lo(c + 1, W, Gc);
-    if (u0 >= u1) return;
-    const int b = find_req(s_pref, a.B, u1 - 1);
-    const ReqInfo ri = info[b];
-    const long long local = u1 - 1 - s_pref[b];
-    const int seg = (int)(local / ri.nt);
-    const long long seg_start = s_pref[b] + (long long)seg * ri.nt;
-    const long long seg_end = seg_start + ri.nt;
-    if (!(seg_start >= u0 && seg_end > u1)) return;  // not the first owner of a split segment
+    const int c = blockIdx.x;
+    const CombJob job = a.jobs[c];
+    if (job.b < 0) return;
     const int G = a.Hq / a.Hkv;
-    const int n0 = a.node_off[b];
-    const int N = a.node_off[b + 1] - n0;
-    const int kvh = seg / ri.mt, mtile = seg - kvh * ri.mt;
+    const int n0 = job.n0, N = job.N, kvh = job.kvh, mtile = job.mtile;
     const int r0 = blockIdx.y * kCombRows;
     const int rows = min(kCombRows, N * G - mtile * kBM - r0);
     if (rows <= 0) return;
-    const long long c1 = owner_of(seg_end - 1, W, Gc);
-    if (threadIdx.x == 0) {
-        int np = 0;
-        for (long long cc = c; cc <= c1 && np < kMaxPieces; ++cc) {
-            const long long lo = range_lo(cc, W, Gc);
-            if (lo == range_lo(cc + 1, W, Gc)) continue;  // empty range: no piece
-            s_slot[np++] = (int)(2 * cc + (seg_start > lo ? 1 : 0));
+    const long long Gc = gridDim.x;
+    int np;
+    if (job.W >= Gc) {  // every range is non-empty: one piece per CTA c .. c1
+        np = job.c1 - c + 1;
+        for (int x = threadIdx.x; x < np; x += kCombThreads) s_slot[x] = x == 0 ? job.first_slot : 2 * (c + x);
+    } else {
+        __shared__ int s_np;
+        if (threadIdx.x == 0) {
+            int n = 0;
+            s_slot[n++] = job.first_slot;
+            for (long long cc = c + 1; cc <= job.c1 && n < kAttnMaxGrid; ++cc)
+                if (range_lo(cc, job.W, Gc) < range_lo(cc + 1, job.W, Gc)) s_slot[n++] = (int)(2 * cc);
+            s_np = n;
         }
-        s_np = np;
+        __syncthreads();
+        np = s_np;
     }
     __syncthreads();
-    const int np = s_np;
     const int D = a.D;
+
+    // phase-2 items of this thread (row, column quad), and the first batch of
+    // their partial loads, issued before phase 1 so both share one round trip
+    constexpr int kMaxItems = kCombRows * 128 / 4 / kCombThreads;  // 4 for D = 128
+    const int d4 = D / 4;
+    const int nitems = rows * d4;
+    float4 acc[kMaxItems];
+    int irow[kMaxItems];
+#pragma unroll
+    for (int k = 0; k < kMaxItems; ++k) {
+        acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        const int x = threadIdx.x + k * kCombThreads;
+        irow[k] = x < nitems ? x / d4 : -1;
+    }
+    float m[kCombBatch][kMaxItems];
+    float4 o[kCombBatch][kMaxItems];
+    auto load_batch = [&](int p0) {
+#pragma unroll
+        for (int q = 0; q < kCombBatch; ++q) {
+            const long long base = p0 + q < np ? (long long)s_slot[p0 + q] * kBM + r0 : -1;
+#pragma unroll
+            for (int k = 0; k < kMaxItems; ++k) {
+                m[q][k] = -INFINITY;
+                o[q][k] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (base >= 0 && irow[k] >= 0) {
+                    const int x = threadIdx.x + k * kCombThreads;
+                    const int r = irow[k], cq = x - r * d4;
+                    m[q][k] = a.part_m[base + r];
+                    o[q][k] = *reinterpret_cast<const float4 *>(a.part_o + (base + r) * D + cq * 4);
+                }
+            }
+        }
+    };
+    load_batch(0);
 
     // phase 1: per-row M and 1 / L
     {
@@ -144,13 +175,13 @@ attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
         if (r < rows) {
             for (int p = j; p < np; p += kCombFold) {
                 const long long prow = (long long)s_slot[p] * kBM + r0 + r;
-                const float m = a.part_m[prow], l = a.part_l[prow];
-                if (m == -INFINITY) continue;
-                if (m > fm) {
-                    fl = fl * __expf(fm - m) + l;  // fm = -inf: fl = 0
-                    fm = m;
+                const float mp = a.part_m[prow], lp = a.part_l[prow];
+                if (mp == -INFINITY) continue;
+                if (mp > fm) {
+                    fl = fl * __expf(fm - mp) + lp;  // fm = -inf: fl = 0
+                    fm = mp;
                 } else {
-                    fl += l * __expf(m - fm);
+                    fl += lp * __expf(mp - fm);
                 }
             }
         }
@@ -176,36 +207,9 @@ attn_combine(AttnArgs a, const ReqInfo *__restrict__ info) {
         __syncthreads();
     }
 
-    // phase 2: the weighted sum of the partial outputs
-    constexpr int kMaxItems = kCombRows * 128 / 4 / kCombThreads;  // 4 for D = 128
-    const int d4 = D / 4;
-    const int nitems = rows * d4;
-    float4 acc[kMaxItems];
-    int irow[kMaxItems];
-#pragma unroll
-    for (int k = 0; k < kMaxItems; ++k) {
-        acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-        const int x = threadIdx.x + k * kCombThreads;
-        irow[k] = x < nitems ? x / d4 : -1;
-    }
+    // phase 2: the weighted sum of the partial outputs, kCombBatch pieces a round
     for (int p0 = 0; p0 < np; p0 += kCombBatch) {
-        float m[kCombBatch][kMaxItems];
-        float4 o[kCombBatch][kMaxItems];
-#pragma unroll
-        for (int q = 0; q < kCombBatch; ++q) {
-            const long long base = p0 + q < np ? (long long)s_slot[p0 + q] * kBM + r0 : -1;
-#pragma unroll
-            for (int k = 0; k < kMaxItems; ++k) {
-                m[q][k] = -INFINITY;
-                o[q][k] = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (base >= 0 && irow[k] >= 0) {
-                    const int x = threadIdx.x + k * kCombThreads;
-                    const int r = irow[k], cq = x - r * d4;
-                    m[q][k] = a.part_m[base + r];
-                    o[q][k] = *reinterpret_cast<const float4 *>(a.part_o + (base + r) * D + cq * 4);
-                }
-            }
-        }
+        if (p0 > 0) load_batch(p0);
 #pragma unroll
         for (int q = 0; q < kCombBatch; ++q) {
 #pragma unroll
@@ -269,7 +273,7 @@ int g_attr_done[64][2] = {};
 
 using namespace rs;
 
-static int attn_grid() { return num_sms(); }
+static int attn_grid() { return std::min(num_sms(), kAttnMaxGrid); }
 
 extern "C" size_t rs_tree_verify_attn_workspace_size(int B, int R, int Hq, int Hkv, int D) {
     if (B < 0 || R < 0 || Hq < 1 || Hkv < 1 || (D != 64 && D != 128)) return 0;
@@ -280,6 +284,7 @@ extern "C" size_t rs_tree_verify_attn_workspace_size(int B, int R, int Hq, int H
     cv.take<float>(2 * Gc * kBM * (size_t)D);
     cv.take<float>(2 * Gc * kBM);
     cv.take<float>(2 * Gc * kBM);
+    cv.take<CombJob>(Gc);
     return cv.used();
 }
 
@@ -325,6 +330,7 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     a.part_o = cv.take<float>(2 * (size_t)Gc * kBM * D);
     a.part_m = cv.take<float>(2 * (size_t)Gc * kBM);
     a.part_l = cv.take<float>(2 * (size_t)Gc * kBM);
+    a.jobs = cv.take<CombJob>((size_t)Gc);
     a.B = B;
     a.Hq = Hq;
     a.Hkv = Hkv;
@@ -368,7 +374,7 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     else
         attn_tc_kernel<64><<<Gc, kAttnThreads, smem, st>>>(a, info, tmk, tmv);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/main");
-    attn_combine<<<dim3(Gc, kCombGroups), kCombThreads, (size_t)(B + 1) * sizeof(int), st>>>(a, info);
+    attn_combine<<<dim3(Gc, kCombGroups), kCombThreads, 0, st>>>(a);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/combine");
     return RS_OK;
 }

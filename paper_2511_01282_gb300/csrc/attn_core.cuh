@@ -52,6 +52,7 @@ constexpr int kNumBars = 4 * kNS + 12;
 constexpr int kSmemMisc = kSmemBar + kNumBars * 8;  // tmem base, abort flag
 constexpr int kSmemPref = kSmemMisc + 16;
 constexpr int kAttnMaxB = 4096;
+constexpr int kAttnMaxGrid = 256;  // CTAs (one per SM, at most this many)
 constexpr long long kWaitLimit = 4000000000ll;     // clock cycles (~2 s)
 constexpr uint32_t kTmemCols = 512;
 // TMEM columns: O [0, 128), S/P buffers [128, 256) and [256, 384), Q [384, 448)
@@ -66,12 +67,25 @@ struct ReqInfo {
     int ok;
 };
 
+// The split segment a CTA starts, for attn_combine: the segment that begins
+// in the CTA's range and continues past it (at most one per CTA).
+struct CombJob {
+    long long W;     // units of the launch
+    int b;           // request (-1: the CTA starts no split segment)
+    int kvh, mtile;  // the segment's KV head and row tile
+    int n0, N;       // the request's first node and node count
+    int first_slot;  // partial slot of the segment's first piece
+    int c1;          // last CTA holding a piece of the segment
+    int pad;
+};
+
 struct AttnArgs {
     const uint16_t *q;
     const int64_t *kv_off;
     const int32_t *ctx_len, *node_off;
     const uint32_t *anc;
     float *part_o, *part_m, *part_l;
+    CombJob *jobs;  // [gridDim.x]
     int B, Hq, Hkv, D;
     float scale;
     float *out, *lse;
@@ -138,6 +152,7 @@ struct Piece {
     bool final;                  // the piece is the whole segment
     int slot;                    // partial slot when not final
     long long end;               // unit index after the piece
+    long long seg_start, seg_end;  // units of the whole segment
 };
 
 __device__ __forceinline__ Piece piece_at(const ReqInfo *__restrict__ info, const int *s_pref, int B,
@@ -156,6 +171,8 @@ __device__ __forceinline__ Piece piece_at(const ReqInfo *__restrict__ info, cons
     pc.j1 = pc.j0 + (int)(pc.end - u);
     pc.final = (seg_start >= u0 && seg_end <= u1);
     pc.slot = (int)(2 * c + (seg_start > u0 ? 1 : 0));
+    pc.seg_start = seg_start;
+    pc.seg_end = seg_end;
     return pc;
 }
 
@@ -288,6 +305,25 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                     mbar_wait(&vfull[t % kNS], (uint32_t)((t / kNS) & 1), &no_abort, kWaitLimit);
                 }
             }
+        }
+        __syncwarp();
+        if (lane == 1) {  // after the producer loop: off the critical path
+            // the split segment this CTA starts (its last piece, when that piece
+            // begins inside the range and ends past it), for attn_combine
+            CombJob job{W, -1, 0, 0, 0, 0, 0, 0, 0};
+            if (u0 < u1) {
+                const Piece pl = piece_at(info, s_pref, a.B, u1 - 1, u0, u1, c);
+                if (pl.seg_start >= u0 && pl.seg_end > u1) {
+                    job.b = pl.b;
+                    job.kvh = pl.kvh;
+                    job.mtile = pl.mtile;
+                    job.n0 = a.node_off[pl.b];
+                    job.N = a.node_off[pl.b + 1] - job.n0;
+                    job.first_slot = (int)(2 * c + (pl.seg_start > u0 ? 1 : 0));
+                    job.c1 = (int)owner_of(pl.seg_end - 1, W, Gc);
+                }
+            }
+            a.jobs[c] = job;
         }
     } else if (warp == kMmaWarp) {
         // ---------------------------------------------------------- MMA issuer
