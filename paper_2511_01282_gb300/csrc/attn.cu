@@ -339,6 +339,7 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     a.out = out;
     a.lse = lse;
     a.status = status;
+    a.kv_stream = 2.0 * (double)kv_rows * Hkv * D * 2 > 0.5 * (double)l2_bytes();
     cudaStream_t st = (cudaStream_t)stream;
 
     // a map over an empty KV cache is never dereferenced: point it at q

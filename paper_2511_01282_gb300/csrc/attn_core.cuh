@@ -86,6 +86,7 @@ struct AttnArgs {
     const uint32_t *anc;
     float *part_o, *part_m, *part_l;
     CombJob *jobs;  // [gridDim.x]
+    int kv_stream;  // the launch's K/V is large next to L2: stream tiles read once
     int B, Hq, Hkv, D;
     float scale;
     float *out, *lse;
@@ -276,9 +277,14 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
         if (lane == 0) {
             long long g = 0;
             bool ok = true;
+            // K/V of a segment with a single row tile is read once per launch;
+            // when the launch's K/V is large next to L2 it is streamed with
+            // evict-first, so it does not push the rest out of L2
+            const uint64_t once = l2_evict_first_policy();
             for (long long u = u0; u < u1 && ok;) {
                 const Piece pc = piece_at(info, s_pref, a.B, u, u0, u1, c);
                 const long long kv0 = a.kv_off[pc.b];
+                const bool reread = !a.kv_stream || info[pc.b].mt > 1;  // kept in L2
                 for (int jt = pc.j0; jt < pc.j1; ++jt, ++g) {
                     const int st = (int)(g % kNS);
                     const uint32_t free_par = (uint32_t)(((g / kNS) & 1) ^ 1);
@@ -289,11 +295,17 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                     if (!(ok = mbar_wait(&kempty[st], free_par, s_abort, kWaitLimit))) break;
                     mbar_expect_tx(&kfull[st], kTileTx);
 #pragma unroll
-                    for (int kb = 0; kb < kKB; ++kb) tma_load_3d(sk + kb * 16384, &tmk, &kfull[st], kb * 64, pc.kvh, row);
+                    for (int kb = 0; kb < kKB; ++kb) {
+                        if (reread) tma_load_3d(sk + kb * 16384, &tmk, &kfull[st], kb * 64, pc.kvh, row);
+                        else tma_load_3d_hint(sk + kb * 16384, &tmk, &kfull[st], kb * 64, pc.kvh, row, once);
+                    }
                     if (!(ok = mbar_wait(&vempty[st], free_par, s_abort, kWaitLimit))) break;
                     mbar_expect_tx(&vfull[st], kTileTx);
 #pragma unroll
-                    for (int kb = 0; kb < kKB; ++kb) tma_load_3d(sv + kb * 16384, &tmv, &vfull[st], kb * 64, pc.kvh, row);
+                    for (int kb = 0; kb < kKB; ++kb) {
+                        if (reread) tma_load_3d(sv + kb * 16384, &tmv, &vfull[st], kb * 64, pc.kvh, row);
+                        else tma_load_3d_hint(sv + kb * 16384, &tmv, &vfull[st], kb * 64, pc.kvh, row, once);
+                    }
                 }
                 u = pc.end;
             }

@@ -35,6 +35,20 @@ int num_sms() {
     return cache[dev];
 }
 
+long long l2_bytes() {
+    static std::mutex mu;
+    static long long cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 128ll << 20;
+    std::lock_guard<std::mutex> lk(mu);
+    if (!cache[dev]) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrL2CacheSize, dev) != cudaSuccess || n <= 0) n = 128 << 20;
+        cache[dev] = n;
+    }
+    return cache[dev];
+}
+
 }  // namespace rs
 
 extern "C" {

@@ -53,6 +53,7 @@ struct Carve {
 };
 
 int num_sms();  // SM count of the current device (cached per device)
+long long l2_bytes();  // L2 size of the current device (cached per device)
 
 // ---------------------------------------------------------------- device side
 __device__ __forceinline__ float warp_max(float v) {
