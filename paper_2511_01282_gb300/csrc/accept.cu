@@ -326,6 +326,7 @@ template <bool kVec, bool kEnt>
 __global__ void __launch_bounds__(kAccThreads, 3)
 accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, int n_items,
             VI *__restrict__ cand, MS *__restrict__ part) {
+    pdl_enter();
     __shared__ RowsShared sh[2];
     extern __shared__ __align__(16) float s_stage[];  // kRowsStages x kAccChunk
     const int step = gridDim.x;
@@ -356,6 +357,7 @@ __global__ void __launch_bounds__(kMergeThreads)
 accept_merge(const VI *__restrict__ cand, const MS *__restrict__ part, int nchunks, int beta, int R,
              int32_t *__restrict__ argmax, int32_t *__restrict__ topk, float *__restrict__ lse,
              float *__restrict__ entropy, float *__restrict__ rowmax) {
+    pdl_enter();
     const int lane = threadIdx.x & 31;
     const long long r = (long long)blockIdx.x * (kMergeThreads / 32) + (threadIdx.x >> 5);
     if (r >= R) return;
@@ -418,6 +420,7 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
               int32_t *__restrict__ acc_len, int32_t *__restrict__ acc_nodes, int32_t *__restrict__ bonus,
               int32_t *__restrict__ winner, uint8_t *__restrict__ commit, float *__restrict__ scores,
               int32_t *__restrict__ status) {
+    pdl_enter();
     const int b = blockIdx.x;
     const int n0 = node_off[b];
     const int N = node_off[b + 1] - n0;
@@ -752,22 +755,26 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
             attr_done[dev] = 1;
         }
         if (vec && ent)
-            accept_rows<true, true><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, n_items, cand, part);
+            launch_full(accept_rows<true, true>, dim3(grid), dim3(kAccThreads), kRowsSmem, st, logits, V, nchunks,
+                p.beta, n_items, cand, part);
         else if (vec)
-            accept_rows<true, false><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, n_items, cand, part);
+            launch_full(accept_rows<true, false>, dim3(grid), dim3(kAccThreads), kRowsSmem, st, logits, V,
+                nchunks, p.beta, n_items, cand, part);
         else if (ent)
-            accept_rows<false, true><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, n_items, cand, part);
+            launch_full(accept_rows<false, true>, dim3(grid), dim3(kAccThreads), kRowsSmem, st, logits, V,
+                nchunks, p.beta, n_items, cand, part);
         else
-            accept_rows<false, false><<<grid, kAccThreads, kRowsSmem, st>>>(logits, V, nchunks, p.beta, n_items, cand, part);
+            launch_full(accept_rows<false, false>, dim3(grid), dim3(kAccThreads), kRowsSmem, st, logits, V,
+                nchunks, p.beta, n_items, cand, part);
         RS_CHECK_LAUNCH("rs_accept/accept_rows");
-        accept_merge<<<(R + kMergeThreads / 32 - 1) / (kMergeThreads / 32), kMergeThreads, 0, st>>>(
-            cand, part, nchunks, p.beta, R, argmax, topk, lse, entropy, rowmax);
+        launch_pdl(accept_merge, dim3((R + kMergeThreads / 32 - 1) / (kMergeThreads / 32)), dim3(kMergeThreads),
+            0, st, cand, part, nchunks, p.beta, R, argmax, topk, lse, entropy, rowmax);
         RS_CHECK_LAUNCH("rs_accept/accept_merge");
     }
     if (B > 0) {
-        accept_decide<<<B, kDecThreads, 0, st>>>(logits, V, node_off, tokens, parents, source, chain, sel_pos,
-                                                 tok_off, p, acc_cap, argmax, topk, lse, rowmax, p_tok, acc_len,
-                                                 acc_nodes, bonus, winner, commit, scores, status);
+        launch_pdl(accept_decide, dim3(B), dim3(kDecThreads), 0, st, logits, V, node_off, tokens, parents,
+            source, chain, sel_pos, tok_off, p, acc_cap, argmax, topk, lse, rowmax, p_tok, acc_len, acc_nodes,
+            bonus, winner, commit, scores, status);
         RS_CHECK_LAUNCH("rs_accept/accept_decide");
     }
     return RS_OK;

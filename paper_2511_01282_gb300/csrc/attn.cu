@@ -35,6 +35,7 @@ attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_
           const int32_t *__restrict__ parents, int Hq, int Hkv, int D, ReqInfo *__restrict__ info,
           uint32_t *__restrict__ anc, float *__restrict__ out, float *__restrict__ lse,
           int32_t *__restrict__ status) {
+    pdl_enter();
     const int b = blockIdx.x, tid = threadIdx.x;
     const int n0 = node_off[b];
     const int N = node_off[b + 1] - n0;
@@ -103,6 +104,7 @@ constexpr int kCombBatch = 2;                    // pieces per phase-2 round
 
 __global__ void __launch_bounds__(kCombThreads, 4)  // the 4 x Gc blocks in one wave
 attn_combine(AttnArgs a) {
+    pdl_enter();
     __shared__ int s_slot[kAttnMaxGrid];
     __shared__ float s_fm[kCombFold][kCombRows], s_fl[kCombFold][kCombRows];
     __shared__ float s_M[kCombRows], s_iL[kCombRows];
@@ -351,7 +353,8 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
         return RS_ERR_CUDA;
     }
 
-    attn_prep<<<B, 256, 0, st>>>(node_off, ctx_len, parents, Hq, Hkv, D, info, anc, out, lse, status);
+    launch_pdl(attn_prep, dim3(B), dim3(256), 0, st, node_off, ctx_len, parents, Hq, Hkv, D, info, anc, out, lse,
+        status);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/prep");
 
     int dev = 0;
@@ -371,11 +374,11 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     }
     const size_t smem = attn_smem_bytes(B);
     if (D == 128)
-        attn_tc_kernel<128><<<Gc, kAttnThreads, smem, st>>>(a, info, tmk, tmv);
+        launch_full(attn_tc_kernel<128>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
     else
-        attn_tc_kernel<64><<<Gc, kAttnThreads, smem, st>>>(a, info, tmk, tmv);
+        launch_full(attn_tc_kernel<64>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/main");
-    attn_combine<<<dim3(Gc, kCombGroups), kCombThreads, 0, st>>>(a);
+    launch_pdl(attn_combine, dim3(Gc, kCombGroups), dim3(kCombThreads), 0, st, a);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/combine");
     return RS_OK;
 }

@@ -221,6 +221,7 @@ template <int D>
 __global__ void __launch_bounds__(kAttnThreads, 1)
 attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_constant__ CUtensorMap tmk,
                const __grid_constant__ CUtensorMap tmv) {
+    pdl_launch_next();
     using namespace sm100;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -262,6 +263,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
         prefetch_tmap(&tmk);
         prefetch_tmap(&tmv);
     }
+    pdl_wait_prev();  // the prologue above touches no global memory
     unit_prefix(info, a.B, s_pref);  // contains __syncthreads
     tc_fence_after();
     const uint32_t tmem = *s_tmem;

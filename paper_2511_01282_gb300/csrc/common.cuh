@@ -35,6 +35,35 @@ void count_launch(int n = 1);
         ::rs::count_launch();                                                        \
     } while (0)
 
+// Kernels are launched with programmatic stream serialization: the next
+// kernel in the stream may begin launching as soon as every block of this one
+// has started (pdl_enter's first instruction), and each kernel waits for its
+// predecessor's completion and memory before it touches global memory (its
+// second).  Since every kernel waits, completion stays ordered along the
+// whole stream.  Without a programmatic predecessor the wait returns at once.
+// Persistent kernels, whose grid assumes every SM free, use launch_full
+// instead: they start only once the previous kernel has finished.
+template <bool kEarly = true, typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = kEarly ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+template <typename... KArgs, typename... Args>
+cudaError_t launch_full(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                        Args... args) {
+    return launch_pdl<false>(kern, grid, block, smem, st, args...);
+}
+
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Bump allocator over the caller's workspace (256-byte aligned slices).
@@ -56,6 +85,14 @@ int num_sms();  // SM count of the current device (cached per device)
 long long l2_bytes();  // L2 size of the current device (cached per device)
 
 // ---------------------------------------------------------------- device side
+// Let the next kernel start launching, then wait for the previous kernel.
+__device__ __forceinline__ void pdl_launch_next() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait_prev() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_enter() {
+    pdl_launch_next();
+    pdl_wait_prev();
+}
+
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));

@@ -58,6 +58,7 @@ __device__ __forceinline__ float ex2f_approx(float x) {
 template <bool kVec>
 __global__ void __launch_bounds__(kGateThreads)
 entropy_partial(const float *__restrict__ logits, int V, int nchunks, Ent3 *__restrict__ part) {
+    pdl_enter();
     const long long blk = blockIdx.x;
     const long long r = blk / nchunks;
     const int chunk = (int)(blk - r * nchunks);
@@ -135,6 +136,7 @@ constexpr int kMergeThreads = 256;
 
 __global__ void __launch_bounds__(kMergeThreads)
 entropy_merge(const Ent3 *__restrict__ part, int nchunks, int R, float *__restrict__ entropy) {
+    pdl_enter();
     const int lane = threadIdx.x & 31;
     const long long r = (long long)blockIdx.x * (kMergeThreads / 32) + (threadIdx.x >> 5);
     if (r >= R) return;
@@ -182,6 +184,7 @@ gate_push(const float *__restrict__ entropy, const int32_t *__restrict__ row_off
           const uint8_t *__restrict__ row_commit, rs_params p, float *__restrict__ hist,
           int32_t *__restrict__ hist_n, int32_t *__restrict__ k_star, float *__restrict__ h_best,
           uint8_t *__restrict__ entropy_ok) {
+    pdl_enter();
     const int b = blockIdx.x, tid = threadIdx.x;
     const int r0 = row_off[b], r1 = row_off[b + 1];
     const int l = p.l;
@@ -259,17 +262,19 @@ rs_status launch_gate(const char *who, const float *logits, int R, int V, int nc
         }
         const bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
         if (vec)
-            entropy_partial<true><<<(unsigned)blocks, kGateThreads, 0, st>>>(logits, V, nchunks, part);
+            launch_pdl(entropy_partial<true>, dim3((unsigned)blocks), dim3(kGateThreads), 0, st, logits, V,
+                nchunks, part);
         else
-            entropy_partial<false><<<(unsigned)blocks, kGateThreads, 0, st>>>(logits, V, nchunks, part);
+            launch_pdl(entropy_partial<false>, dim3((unsigned)blocks), dim3(kGateThreads), 0, st, logits, V,
+                nchunks, part);
         RS_CHECK_LAUNCH(who);
-        entropy_merge<<<(R + kMergeThreads / 32 - 1) / (kMergeThreads / 32), kMergeThreads, 0, st>>>(
-            part, nchunks, R, entropy);
+        launch_pdl(entropy_merge, dim3((R + kMergeThreads / 32 - 1) / (kMergeThreads / 32)), dim3(kMergeThreads),
+            0, st, part, nchunks, R, entropy);
         RS_CHECK_LAUNCH(who);
     }
     if (B > 0) {
-        gate_push<<<B, kPushThreads, 0, st>>>(entropy, row_off, row_commit, p, hist, hist_n, k_star, h_best,
-                                              entropy_ok);
+        launch_pdl(gate_push, dim3(B), dim3(kPushThreads), 0, st, entropy, row_off, row_commit, p, hist, hist_n,
+            k_star, h_best, entropy_ok);
         RS_CHECK_LAUNCH(who);
     }
     return RS_OK;
@@ -386,8 +391,8 @@ extern "C" rs_status rs_entropy_gate_rows(const float *entropy, const int32_t *r
     RS_CHECK_ARG(B == 0 || (entropy && row_off && row_commit && hist && hist_n && k_star && h_best && entropy_ok),
                  "rs_entropy_gate_rows: null pointer");
     if (B == 0) return RS_OK;
-    gate_push<<<B, kPushThreads, 0, (cudaStream_t)stream>>>(entropy, row_off, row_commit, p, hist, hist_n, k_star,
-                                                            h_best, entropy_ok);
+    launch_pdl(gate_push, dim3(B), dim3(kPushThreads), 0, (cudaStream_t)stream, entropy, row_off, row_commit, p,
+        hist, hist_n, k_star, h_best, entropy_ok);
     RS_CHECK_LAUNCH("rs_entropy_gate_rows");
     return RS_OK;
 }

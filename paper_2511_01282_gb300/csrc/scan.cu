@@ -199,6 +199,7 @@ match_scan_kernel(const int32_t *__restrict__ tokens, const int64_t *__restrict_
                   int32_t *__restrict__ count, int32_t *__restrict__ pos, int32_t *__restrict__ sel_pos,
                   int32_t *__restrict__ sel_len, int32_t *__restrict__ spans, int32_t *__restrict__ n_sel,
                   int32_t *__restrict__ status) {
+    pdl_enter();
     cg::cluster_group cluster = cg::this_cluster();
     const int crank = (int)cluster.block_rank();
     const int b = blockIdx.y;
@@ -492,9 +493,9 @@ extern "C" rs_status rs_match_scan(const int32_t *tokens, const int64_t *tok_off
         }
         attr_done[dev] = 1;
     }
-    match_scan_kernel<<<dim3(kScanCluster, B), kScanThreads, sizeof(ScanShared), (cudaStream_t)stream>>>(
-        tokens, tok_off, k_star, gate_ok, scores, p.theta_score, p.top_c, p.span_len, pos_cap, count, pos,
-        sel_pos, sel_len, spans, n_sel, status);
+    launch_pdl(match_scan_kernel, dim3(kScanCluster, B), dim3(kScanThreads), sizeof(ScanShared),
+        (cudaStream_t)stream, tokens, tok_off, k_star, gate_ok, scores, p.theta_score, p.top_c, p.span_len,
+        pos_cap, count, pos, sel_pos, sel_len, spans, n_sel, status);
     RS_CHECK_LAUNCH("rs_match_scan");
     return RS_OK;
 }
