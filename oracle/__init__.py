@@ -44,6 +44,11 @@ def lib():
         L.rsref_accept.argtypes = ([P, C.c_long, P, C.c_int, P, P, P, P, P, C.c_int, P,
                                     C.c_int, C.c_double, C.c_int, C.c_int, C.c_double,
                                     C.c_int] + [P] * 11)
+        L.rsref_sample_row.restype = C.c_int
+        L.rsref_sample_row.argtypes = [P, C.c_long, C.c_double, C.c_double]
+        L.rsref_tree_sample.restype = None
+        L.rsref_tree_sample.argtypes = ([P, C.c_long, P, C.c_int, P, P, P, C.c_double, P, C.c_int]
+                                        + [P] * 5)
         _lib = L
     return _lib
 
@@ -188,6 +193,30 @@ def accept(logits, node_off, tokens, parents, source, chain, sel_pos, tok_off, s
                        _p(out["bonus"]), _p(out["winner"]), _p(out["commit"]), _p(scores),
                        _p(out["status"]))
     out["scores"] = scores
+    return out
+
+
+# ---------------------------------------------------------------- sampling
+def sample_row(z, T, u):
+    """Section 3.4 drafter outputs: the inverse-CDF draw (token-id order) from softmax(z/T)."""
+    z = _c(z, np.float32)
+    return int(lib().rsref_sample_row(_p(z), z.size, float(T), float(u)))
+
+
+def tree_sample(logits, node_off, tokens, parents, source, T, u, acc_cap):
+    """Per-row draws and the lossless walk over the model-drafted nodes."""
+    logits = _c(logits, np.float32)
+    R, V = logits.shape
+    node_off = _c(node_off, np.int32)
+    B = node_off.size - 1
+    u = _c(u, np.float64)
+    out = dict(draw=np.empty(R, np.int32), acc_len=np.empty(B, np.int32),
+               acc_nodes=np.empty((B, acc_cap), np.int32), bonus=np.empty(B, np.int32),
+               status=np.empty(B, np.int32))
+    lib().rsref_tree_sample(_p(logits), V, _p(node_off), B, _p(_c(tokens, np.int32)),
+                            _p(_c(parents, np.int32)), _p(_c(source, np.uint8)), float(T), _p(u),
+                            acc_cap, _p(out["draw"]), _p(out["acc_len"]), _p(out["acc_nodes"]),
+                            _p(out["bonus"]), _p(out["status"]))
     return out
 
 

@@ -10,7 +10,7 @@ import subprocess
 import sys
 
 HERE = os.path.dirname(os.path.abspath(__file__))
-SOURCES = ["entropy.c", "match.c", "attn.c", "accept.c"]
+SOURCES = ["entropy.c", "match.c", "attn.c", "accept.c", "sample.c"]
 LIB = os.path.join(HERE, "librsref.so")
 
 

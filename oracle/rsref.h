@@ -100,6 +100,24 @@ void rsref_accept(const float *logits, long V, const int *node_off, int B,
                   int *acc_len, int *acc_nodes, int *bonus, int *winner,
                   unsigned char *commit, float *scores, int *status);
 
+/* ---- Section 3.4, drafter outputs: lossless speculative sampling ------- */
+/* The draw from one row at temperature T > 0 for a uniform u in [0, 1): the
+ * smallest token id v with sum_{w <= v} p_T(w) > u, where p_T = softmax(z/T)
+ * (the inverse CDF in token-id order).  Rows without mass give 0. */
+int rsref_sample_row(const float *z, long V, double T, double u);
+
+/* draw[r] = rsref_sample_row(row r, u[r]) for every node row; then per
+ * request, from the root: while a model child (source 1) of the current node
+ * carries the current node's draw, accept it (acc_nodes, in depth order) and
+ * move to it; the first draw without such a child is the correction token
+ * (bonus).  acc_len counts every accepted node (TRUNCATED when more than
+ * acc_cap); a malformed tree gives BAD_TREE, acc_len 0, bonus -1. */
+void rsref_tree_sample(const float *logits, long V, const int *node_off, int B,
+                       const int *tokens, const int *parents,
+                       const unsigned char *source, double T, const double *u,
+                       int acc_cap, int *draw, int *acc_len, int *acc_nodes,
+                       int *bonus, int *status);
+
 #ifdef __cplusplus
 }
 #endif
