@@ -336,7 +336,8 @@ def run_ours(args, rank, world, local_rank):
     call_ms = {"gate_rows": time_call(st.gate_rows, n_call),
                "scan": time_call(lambda sm: st.scan(stream=sm), n_call),
                "attn": time_call(st.attn, n_call), "accept": time_call(lambda sm: st.accept(stream=sm), n_call),
-               "gate_from_logits": time_call(st.gate, n_call)}
+               "gate_from_logits": time_call(st.gate, n_call),
+               "tree_sample": time_call(lambda sm: st.tree_sample(1.0, sm), n_call)}
     st.reset_state()
     torch.cuda.synchronize()
 

@@ -286,6 +286,46 @@ rs_status rs_accept(const float *logits, int R, int V, const int32_t *node_off, 
                     int32_t *bonus, int32_t *winner, uint8_t *commit, float *scores,
                     int32_t *status, void *workspace, size_t workspace_bytes, void *stream);
 
+/* ======================================================= rs_tree_sample ===
+ * Section 3.4, "For Drafter Module outputs": lossless speculative sampling
+ * of the model-drafted nodes (the non-greedy counterpart of rs_accept's
+ * strict check).  The model children of a node are deterministic expansions
+ * (a point-mass proposal each); speculative sampling over them has the law
+ * of: draw y from the target row at temperature T, accept the model child
+ * carrying y and continue from it, otherwise y is the correction token.
+ * Every row's draw is the inverse CDF, in token-id order, of the caller's
+ * uniform: the smallest id v with sum_{w <= v} softmax(z / T)(w) > u.
+ * Retrieved nodes (source 2) are not proposals here; they are verified by
+ * rs_accept's relaxed procedure.
+ *
+ *   logits, R, V, node_off, B, tokens, parents, source: as for rs_accept.
+ *   temperature  T > 0 (finite), RS_ERR_INVALID_ARG otherwise.
+ *   uniforms [R] fp32 in [0, 1): one per row, drawn by the caller (e.g. a
+ *            counter-based generator); a value >= 1 selects the row's last
+ *            id with mass.
+ *   acc_cap  capacity of acc_nodes per request (>= 1).
+ * Outputs:
+ *   draw    [R] int32     every row's draw (0 for a row without mass);
+ *   acc_len [B] int32     accepted model nodes from the root (RS_ST_TRUNCATED
+ *                         when above acc_cap: acc_nodes keeps the first ones);
+ *   acc_nodes [B, acc_cap] int32  local node indices in depth order, -1 padded;
+ *   bonus   [B] int32     the correction token (the draw of the last accepted
+ *                         node, or of the root);
+ *   status  [B] int32     RS_ST_BAD_TREE (parents / source layout) or
+ *                         RS_ST_TOO_LARGE (more than RS_MAX_NODES nodes):
+ *                         acc_len 0, bonus -1.
+ * Workspace: rs_tree_sample_workspace_size(R, V) bytes (per 8192-logit chunk
+ * of every row: its maximum and its mass).  Draws are computed in fp32; a
+ * uniform within ~1e-5 relative of a CDF step may land on the neighbouring
+ * token relative to an fp64 evaluation.
+ */
+size_t rs_tree_sample_workspace_size(int R, int V);
+rs_status rs_tree_sample(const float *logits, int R, int V, const int32_t *node_off, int B,
+                         const int32_t *tokens, const int32_t *parents, const uint8_t *source,
+                         float temperature, const float *uniforms, int acc_cap, int32_t *draw,
+                         int32_t *acc_len, int32_t *acc_nodes, int32_t *bonus, int32_t *status,
+                         void *workspace, size_t workspace_bytes, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

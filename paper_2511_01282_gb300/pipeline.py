@@ -9,7 +9,9 @@ stream, the calls of one step of Algorithm 1 in their data-flow order:
       -> rs_match_scan (keyed by k*, gated by the trigger)
       -> rs_tree_verify_attn -> rs_accept (also emits the row entropies)
 
-It computes nothing itself.  Inputs come as host numpy arrays (bf16 as
+``tree_sample`` runs rs_tree_sample, the non-greedy (lossless sampling)
+verification of the model drafts, on the same buffers.  It computes nothing
+itself.  Inputs come as host numpy arrays (bf16 as
 uint16 bit patterns) with the layouts ``include/respec.h`` documents.
 """
 import numpy as np
@@ -28,7 +30,7 @@ class VerifyStep:
               "chain", "sel_pos")
 
     def __init__(self, arrays, p, Hq, Hkv, D, pos_cap=1024, acc_cap=64, device="cuda",
-                 scale=None, pinned_host=False):
+                 scale=None, pinned_host=False, sample_seed=0):
         self.p = p
         self.Hq, self.Hkv, self.D = Hq, Hkv, D
         self.scale = float(D ** -0.5 if scale is None else scale)
@@ -67,7 +69,14 @@ class VerifyStep:
             gate=z(max(rs.rs_entropy_gate_workspace_size(R, V), 256), torch.uint8),
             scan=z(max(rs.rs_match_scan_workspace_size(B), 256), torch.uint8),
             attn=z(max(rs.rs_tree_verify_attn_workspace_size(B, R, Hq, Hkv, D), 256), torch.uint8),
-            accept=z(max(rs.rs_accept_workspace_size(R, V, p.beta), 256), torch.uint8))
+            accept=z(max(rs.rs_accept_workspace_size(R, V, p.beta), 256), torch.uint8),
+            sample=z(max(rs.rs_tree_sample_workspace_size(R, V), 256), torch.uint8))
+        # lossless sampling of the model drafts (rs_tree_sample): one uniform per row
+        gen = torch.Generator(device=dev).manual_seed(sample_seed)
+        self.uniforms = torch.rand(max(R, 1), device=dev, generator=gen)
+        self.sample_out = dict(draw=z(max(R, 1), torch.int32), acc_len=z(B, torch.int32),
+                               acc_nodes=z((B, acc_cap), torch.int32), bonus=z(B, torch.int32),
+                               status=z(B, torch.int32))
 
     # ------------------------------------------------------------ the calls
     def gate(self, stream=None):
@@ -106,6 +115,14 @@ class VerifyStep:
                      o["topk"], o["lse"], o["p_tok"], o["acc_entropy"] if entropy else None,
                      o["acc_len"], o["acc_nodes"], o["bonus"], o["winner"], o["commit"], d["scores"],
                      o["acc_status"], self.ws["accept"], stream)
+
+    def tree_sample(self, temperature=1.0, stream=None):
+        """Lossless sampling verification of the model drafts (non-greedy)."""
+        d, o = self.d, self.sample_out
+        rs.rs_tree_sample(d["logits"], self.R, self.V, d["node_off"], self.B, d["tree_tokens"],
+                          d["parents"], d["source"], temperature, self.uniforms, self.acc_cap,
+                          o["draw"], o["acc_len"], o["acc_nodes"], o["bonus"], o["status"],
+                          self.ws["sample"], stream)
 
     def step(self, stream=None, fused=True):
         """One pass of the whole hot path.

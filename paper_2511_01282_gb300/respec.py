@@ -65,6 +65,9 @@ _SIGS = {
     "rs_accept": (C.c_int, [_P, C.c_int, C.c_int, _P, C.c_int, _P, _P, _P, _P, _P, _P, rs_params,
                             C.c_int, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, C.c_size_t,
                             _P]),
+    "rs_tree_sample_workspace_size": (C.c_size_t, [C.c_int, C.c_int]),
+    "rs_tree_sample": (C.c_int, [_P, C.c_int, C.c_int, _P, C.c_int, _P, _P, _P, C.c_float, _P, C.c_int,
+                                 _P, _P, _P, _P, _P, _P, C.c_size_t, _P]),
     "rs_entropy_gate_rows": (C.c_int, [_P, _P, _P, C.c_int, rs_params, _P, _P, _P, _P, _P, _P]),
 }
 
@@ -185,6 +188,19 @@ def rs_tree_verify_attn(q, k, v, kv_rows, kv_off, ctx_len, node_off, parents, B,
 
 def rs_accept_workspace_size(R, V, beta):
     return int(lib().rs_accept_workspace_size(R, V, beta))
+
+
+def rs_tree_sample_workspace_size(R, V):
+    return int(lib().rs_tree_sample_workspace_size(R, V))
+
+
+def rs_tree_sample(logits, R, V, node_off, B, tokens, parents, source, temperature, uniforms,
+                   acc_cap, draw, acc_len, acc_nodes, bonus, status, workspace, stream=None):
+    wp, wb = _ws(workspace)
+    _check(lib().rs_tree_sample(_ptr(logits), R, V, _ptr(node_off), B, _ptr(tokens),
+                                _ptr(parents), _ptr(source), float(temperature), _ptr(uniforms),
+                                acc_cap, _ptr(draw), _ptr(acc_len), _ptr(acc_nodes), _ptr(bonus),
+                                _ptr(status), wp, wb, _stream(stream)))
 
 
 def rs_accept(logits, R, V, node_off, B, tokens, parents, source, chain, sel_pos, tok_off, p,

@@ -63,6 +63,8 @@ def test_workspace_sizes_are_host_computable(rs):
     assert rs.rs_accept_workspace_size(145, 128256, 5) >= 145 * 16 * 5 * 8
     assert rs.rs_match_scan_workspace_size(4) >= 0
     assert rs.rs_entropy_gate_workspace_size(-1, 10) == 0
+    assert rs.rs_tree_sample_workspace_size(145, 128256) >= 145 * 16 * 8
+    assert rs.rs_tree_sample_workspace_size(3, 0) == 0
 
 
 def _fake(n=1):
@@ -104,6 +106,14 @@ def test_bad_arguments_fail_before_launch(rs):
     st = L.rs_tree_verify_attn(f, C.c_void_p(0x10002), f, 10, f, f, f, f, 1, 1, 4, 4, 128, 0.1, f, f, f, f,
                                1 << 30, None)
     assert st == rs.RS_ERR_INVALID_ARG and "aligned" in rs.rs_last_error()
+    # rs_tree_sample: temperature must be finite and positive; acc_cap >= 1
+    for T in (0.0, -1.0, float("inf"), float("nan")):
+        st = L.rs_tree_sample(f, 1, 10, f, 1, f, f, f, T, f, 4, f, f, f, f, f, f, 1 << 20, None)
+        assert st == rs.RS_ERR_INVALID_ARG and "temperature" in rs.rs_last_error()
+    st = L.rs_tree_sample(f, 1, 10, f, 1, f, f, f, 1.0, f, 0, f, f, f, f, f, f, 1 << 20, None)
+    assert st == rs.RS_ERR_INVALID_ARG
+    st = L.rs_tree_sample(f, 4, 100000, f, 1, f, f, f, 1.0, f, 4, f, f, f, f, f, f, 8, None)
+    assert st == rs.RS_ERR_CAPACITY
     # nothing was launched by any of these
     assert rs.rs_launch_count() == n_launch
 
