@@ -338,6 +338,10 @@ def run_ours(args, rank, world, local_rank):
                "attn": time_call(st.attn, n_call), "accept": time_call(lambda sm: st.accept(stream=sm), n_call),
                "gate_from_logits": time_call(st.gate, n_call),
                "tree_sample": time_call(lambda sm: st.tree_sample(1.0, sm), n_call)}
+    # retrieval from the inverted index (NEXT-4) on the same buffers
+    st.build_index()
+    call_ms["scan_indexed"] = time_call(lambda sm: st.scan(stream=sm, indexed=True), n_call)
+    call_ms["index_build"] = time_call(st.build_index, 3)
     st.reset_state()
     torch.cuda.synchronize()
 

@@ -286,6 +286,37 @@ rs_status rs_accept(const float *logits, int R, int V, const int32_t *node_off, 
                     int32_t *bonus, int32_t *winner, uint8_t *commit, float *scores,
                     int32_t *status, void *workspace, size_t workspace_bytes, void *stream);
 
+/* ============================================ rs_match_index (NEXT-4) ====
+ * An index for Section 3.3's retrieval on long buffers.  Algorithm 1 asks
+ * its suffix automaton two things about the key (the buffer's last
+ * k <= RS_MAX_L tokens): Contains and RetrievePositions.  Both are answered
+ * exactly from an inverted index: for every token id, the ascending list of
+ * positions holding it; the positions holding the key's last token are the
+ * candidates, verified against the key's other tokens.  A query costs
+ * O(occurrences of that token) instead of rs_match_scan's O(t).
+ *
+ * rs_match_index_bytes(B, V, t_total): device bytes of an index over B
+ *   buffers of ids in [0, V) (others share one bucket) with t_total tokens
+ *   in all (tok_off[B] at build time).
+ * rs_match_index_build: indexes tokens[tok_off[b] .. tok_off[b+1]) of every
+ *   request (the index remembers each request's length and offset).  The
+ *   caller owns `index`; nothing in it needs initialising.
+ * rs_match_scan_indexed: rs_match_scan's inputs, outputs and meaning, plus
+ *   V, t_total (as given to the build) and the index.  tok_off may have grown
+ *   since the build (tokens appended at the end of a request's buffer, its
+ *   first token's offset unchanged relative to its own buffer): positions
+ *   at or after the length indexed are tested one by one, so rebuild when
+ *   that tail gets long.  One CTA per request.
+ */
+size_t rs_match_index_bytes(int B, int V, int64_t t_total);
+rs_status rs_match_index_build(const int32_t *tokens, const int64_t *tok_off, int B, int V, int64_t t_total,
+                               void *index, size_t index_bytes, void *stream);
+rs_status rs_match_scan_indexed(const int32_t *tokens, const int64_t *tok_off, int B, const int32_t *k_star,
+                                const uint8_t *gate_ok, const float *scores, rs_params p, int pos_cap,
+                                int32_t *count, int32_t *pos, int32_t *sel_pos, int32_t *sel_len,
+                                int32_t *spans, int32_t *n_sel, int32_t *status, int V, int64_t t_total,
+                                const void *index, size_t index_bytes, void *stream);
+
 /* ======================================================= rs_tree_sample ===
  * Section 3.4, "For Drafter Module outputs": lossless speculative sampling
  * of the model-drafted nodes (the non-greedy counterpart of rs_accept's

@@ -10,8 +10,9 @@ stream, the calls of one step of Algorithm 1 in their data-flow order:
       -> rs_tree_verify_attn -> rs_accept (also emits the row entropies)
 
 ``tree_sample`` runs rs_tree_sample, the non-greedy (lossless sampling)
-verification of the model drafts, on the same buffers.  It computes nothing
-itself.  Inputs come as host numpy arrays (bf16 as
+verification of the model drafts, and ``scan(indexed=True)`` the retrieval
+from the inverted index (``build_index``), on the same buffers.  It computes
+nothing itself.  Inputs come as host numpy arrays (bf16 as
 uint16 bit patterns) with the layouts ``include/respec.h`` documents.
 """
 import numpy as np
@@ -92,13 +93,27 @@ class VerifyStep:
                                 d["hist"], d["hist_n"], o["k_star"], o["h_best"], o["entropy_ok"],
                                 stream)
 
-    def scan(self, k_star=None, gate_ok="gate", stream=None):
+    def scan(self, k_star=None, gate_ok="gate", stream=None, indexed=False):
         d, o = self.d, self.out
         ks = o["k_star"] if k_star is None else k_star
         ok = o["entropy_ok"] if gate_ok == "gate" else gate_ok
+        if indexed:  # from the inverted index (build_index first)
+            rs.rs_match_scan_indexed(d["tokens"], d["tok_off"], self.B, ks, ok, d["scores"], self.p, self.pos_cap,
+                                     o["count"], o["pos"], o["sel_pos"], o["sel_len"], o["spans"], o["n_sel"],
+                                     o["scan_status"], self.V, self.t_total, self.index, stream)
+            return
         rs.rs_match_scan(d["tokens"], d["tok_off"], self.B, ks, ok, d["scores"], self.p, self.pos_cap,
                          o["count"], o["pos"], o["sel_pos"], o["sel_len"], o["spans"], o["n_sel"],
                          o["scan_status"], self.ws["scan"], stream)
+
+    def build_index(self, stream=None):
+        """Inverted index over the token buffers, for scan(indexed=True)."""
+        self.t_total = int(self.host["tok_off"][-1])
+        if getattr(self, "index", None) is None:
+            self.index = torch.empty(rs.rs_match_index_bytes(self.B, self.V, self.t_total), dtype=torch.uint8,
+                                     device=self.device)
+        rs.rs_match_index_build(self.d["tokens"], self.d["tok_off"], self.B, self.V, self.t_total, self.index,
+                                stream)
 
     def attn(self, stream=None):
         d, o = self.d, self.out

@@ -65,6 +65,10 @@ _SIGS = {
     "rs_accept": (C.c_int, [_P, C.c_int, C.c_int, _P, C.c_int, _P, _P, _P, _P, _P, _P, rs_params,
                             C.c_int, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, C.c_size_t,
                             _P]),
+    "rs_match_index_bytes": (C.c_size_t, [C.c_int, C.c_int, C.c_int64]),
+    "rs_match_index_build": (C.c_int, [_P, _P, C.c_int, C.c_int, C.c_int64, _P, C.c_size_t, _P]),
+    "rs_match_scan_indexed": (C.c_int, [_P, _P, C.c_int, _P, _P, _P, rs_params, C.c_int] + [_P] * 7
+                              + [C.c_int, C.c_int64, _P, C.c_size_t, _P]),
     "rs_tree_sample_workspace_size": (C.c_size_t, [C.c_int, C.c_int]),
     "rs_tree_sample": (C.c_int, [_P, C.c_int, C.c_int, _P, C.c_int, _P, _P, _P, C.c_float, _P, C.c_int,
                                  _P, _P, _P, _P, _P, _P, C.c_size_t, _P]),
@@ -188,6 +192,24 @@ def rs_tree_verify_attn(q, k, v, kv_rows, kv_off, ctx_len, node_off, parents, B,
 
 def rs_accept_workspace_size(R, V, beta):
     return int(lib().rs_accept_workspace_size(R, V, beta))
+
+
+def rs_match_index_bytes(B, V, t_total):
+    return int(lib().rs_match_index_bytes(B, V, t_total))
+
+
+def rs_match_index_build(tokens, tok_off, B, V, t_total, index, stream=None):
+    _check(lib().rs_match_index_build(_ptr(tokens), _ptr(tok_off), B, V, t_total, _ptr(index),
+                                      index.numel() * index.element_size(), _stream(stream)))
+
+
+def rs_match_scan_indexed(tokens, tok_off, B, k_star, gate_ok, scores, p, pos_cap, count, pos, sel_pos,
+                          sel_len, spans, n_sel, status, V, t_total, index, stream=None):
+    _check(lib().rs_match_scan_indexed(_ptr(tokens), _ptr(tok_off), B, _ptr(k_star), _ptr(gate_ok),
+                                       _ptr(scores), p, pos_cap, _ptr(count), _ptr(pos), _ptr(sel_pos),
+                                       _ptr(sel_len), _ptr(spans), _ptr(n_sel), _ptr(status), V, t_total,
+                                       _ptr(index), index.numel() * index.element_size(),
+                                       _stream(stream)))
 
 
 def rs_tree_sample_workspace_size(R, V):

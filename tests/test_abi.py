@@ -65,6 +65,8 @@ def test_workspace_sizes_are_host_computable(rs):
     assert rs.rs_entropy_gate_workspace_size(-1, 10) == 0
     assert rs.rs_tree_sample_workspace_size(145, 128256) >= 145 * 16 * 8
     assert rs.rs_tree_sample_workspace_size(3, 0) == 0
+    assert rs.rs_match_index_bytes(4, 32000, 131072) >= 131072 * 4 + 4 * 32002 * 4
+    assert rs.rs_match_index_bytes(4, 0, 10) == 0
 
 
 def _fake(n=1):
@@ -114,6 +116,13 @@ def test_bad_arguments_fail_before_launch(rs):
     assert st == rs.RS_ERR_INVALID_ARG
     st = L.rs_tree_sample(f, 4, 100000, f, 1, f, f, f, 1.0, f, 4, f, f, f, f, f, f, 8, None)
     assert st == rs.RS_ERR_CAPACITY
+    # index: too small a buffer for the index, bad V
+    st = L.rs_match_index_build(f, f, 2, 1000, 100, f, 64, None)
+    assert st == rs.RS_ERR_CAPACITY and "index" in rs.rs_last_error()
+    st = L.rs_match_index_build(f, f, 2, 0, 100, f, 1 << 30, None)
+    assert st == rs.RS_ERR_INVALID_ARG
+    st = L.rs_match_scan_indexed(f, f, 1, f, None, f, rs.params(top_c=9), 4, *([f] * 7), 100, 10, f, 1 << 20, None)
+    assert st == rs.RS_ERR_INVALID_ARG
     # nothing was launched by any of these
     assert rs.rs_launch_count() == n_launch
 
