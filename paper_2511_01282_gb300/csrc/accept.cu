@@ -2,19 +2,12 @@
 // and the look-ahead tolerance procedure), longest accepted path and winner
 // (Algorithm 1 l.13), EMA feedback (Eq. 4-5, Algorithm 1 l.15-22).
 //
-// Kernel 1 (accept_rows): three persistent CTAs per SM walk the (row,
-// 8192-logit chunk) work items; each thread copies the next item's 32
-// logits into a second shared-memory stage (cp.async) while it works on the
-// current item from registers.  Per item the CTA produces the chunk's (max,
-// sum e^(z - max)[, sum e^(z - max) (z - max)]) triple and its beta best
-// (logit, id) pairs in the total order (logit desc, id asc).  The beta-th largest of a warp's 32 lane maxima (warp
-// bitonic sort) bounds the chunk's beta-th largest logit from below, and so
-// does the largest such bound over the warps; the few logits at or above it
-// are appended to shared memory and one warp (rotating over items) ranks them
-// by beta rounds of a "best after the previous winner" warp reduction (exact;
-// with many ties at the bound every warp ranks its own logits and that warp
-// merges the lists).
-// No dynamic register indexing.
+// Kernel 1 (accept_rows): one CTA per (row, 8192-logit chunk) streams the
+// chunk once and produces its (max, sum e^(z - max)[, sum e^(z - max)
+// (z - max)]) triple and its beta best (logit, id) pairs in the total order
+// (logit desc, id asc); the top-beta is exact and sort-free apart from one
+// 16-lane sort that sets the candidate threshold.  No dynamic register
+// indexing.
 // Kernel 2 (accept_merge): one warp per row merges the chunk results into
 // argmax, top-beta, log-sum-exp, the row's largest logit (workspace, for
 // kernel 3) and (optionally) the row entropy.
@@ -95,66 +88,60 @@ __device__ __forceinline__ float group_sort_desc(float x, int lane) {
     return x;
 }
 
-// The warp maximum and the largest over the warp's G-lane groups of the
-// group's beta-th largest lane value (beta <= G).
-template <int G>
-__device__ __forceinline__ void warp_max_and_bound(float mx, int lane, int beta, float *wmax, float *bound) {
-    const float sorted = group_sort_desc<G>(mx, lane);
-    float m = -INFINITY, t = -INFINITY;
-#pragma unroll
-    for (int g = 0; g < 32; g += G) {
-        m = fmaxf(m, __shfl_sync(0xffffffffu, sorted, g));
-        t = fmaxf(t, __shfl_sync(0xffffffffu, sorted, g + beta - 1));
-    }
-    *wmax = m;
-    *bound = t;
-}
+constexpr int kHalves = 2 * kAccThreads / 32;  // half-warps per CTA (16 >= RS_MAX_BETA)
+static_assert(kHalves >= RS_MAX_BETA, "the bound needs beta half-warp maxima");
 
-// cp.async: per-thread asynchronous global -> shared copies.  A thread's
-// wait_group only waits for its own copies, so no wait depends on another
-// thread.
-__device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(sm100::smem_u32(smem)), "l"(gmem) : "memory");
-}
-__device__ __forceinline__ void cp_async4(void *smem, const void *gmem) {
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(sm100::smem_u32(smem)), "l"(gmem) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+struct RowsShared {
+    MS sms[kAccThreads / 32];
+    float hmax[kHalves];
+    VI wtop[kAccThreads / 32][RS_MAX_BETA];  // per-warp lists (tie fallback)
+    VI cbuf[kCandCap];                       // the chunk's candidates
+    int cnt;
+};
 
-// Start copying the logits this thread will hold of work item `item` = (row,
-// chunk) into `stage` (the same slots it later reads; ids >= V are skipped).
-template <bool kVec>
-__device__ __forceinline__ void fetch_item(const float *__restrict__ logits, int V, int nchunks, int item,
-                                           float *stage) {
-    const int r = item / nchunks;
-    const int c0 = (item - r * nchunks) * kAccChunk;
-    const float *row = logits + (long long)r * V;
-    const int tid = threadIdx.x;
+// One CTA per (row, 8192-logit chunk) item: the chunk's (max, sum e^(z -
+// max)[, sum e^(z - max) (z - max)]) triple and its beta best (logit, id)
+// pairs in the order (logit desc, id asc).
+//   * Each thread streams 32 logits into registers (eight 128-bit loads; the
+//     in-range test is dropped for chunks that lie inside the row).
+//   * Every lane exponentiates against its warp's maximum, so a warp's
+//     triple is a plain shuffle sum.
+//   * Top-beta: the sixteen half-warp maxima are logits of sixteen disjoint
+//     parts of the chunk, so the beta-th largest of them (one 16-lane sort)
+//     is a lower bound T on the chunk's beta-th largest logit.  Only logits
+//     >= T can be among the best beta; a lane looks at a group of four only
+//     if the group's maximum clears T, appends the survivors to shared
+//     memory, and warp 0 ranks them by counting (rank = the number of
+//     candidates before it in the total order).  If ties at T overflow the
+//     buffer, every warp ranks its own logits by beta "best after the
+//     previous winner" rounds and warp 0 merges the eight lists (exact too).
+template <bool kVec, bool kEnt>
+__global__ void __launch_bounds__(kAccThreads, 4)
+accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *__restrict__ cand,
+            MS *__restrict__ part) {
+    pdl_enter();
+    __shared__ RowsShared sh;
+    const long long blk = blockIdx.x;
+    const long long r = blk / nchunks;
+    const int c0 = (int)(blk - r * nchunks) * kAccChunk;
+    const float *row = logits + r * (long long)V;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    constexpr float kL2E = 1.4426950408889634f;
+    if (tid == 0) sh.cnt = 0;
+
+    // logit id of register j (ids >= V are padding, held as -inf)
+    auto id_of = [&](int j) -> int {
+        if (kVec) return c0 + ((j >> 2) * kAccThreads + tid) * 4 + (j & 3);
+        return c0 + j * kAccThreads + tid;
+    };
+    float v[kAccVpt];
     if (kVec) {
+        const bool inside = c0 + kAccChunk <= V;
 #pragma unroll
         for (int j = 0; j < kAccVpt / 4; ++j) {
-            const int off = (j * kAccThreads + tid) * 4;
-            if (c0 + off < V) cp_async16(stage + off, row + c0 + off);  // V % 4 == 0: whole float4
-        }
-    } else {
-#pragma unroll
-        for (int j = 0; j < kAccVpt; ++j) {
-            const int off = j * kAccThreads + tid;
-            if (c0 + off < V) cp_async4(stage + off, row + c0 + off);
-        }
-    }
-}
-
-template <bool kVec>
-__device__ __forceinline__ void read_item(const float *stage, int V, int c0, float (&v)[kAccVpt]) {
-    const int tid = threadIdx.x;
-    if (kVec) {
-#pragma unroll
-        for (int j = 0; j < kAccVpt / 4; ++j) {
-            const int off = (j * kAccThreads + tid) * 4;
+            const int off = c0 + (j * kAccThreads + tid) * 4;
             float4 x = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
-            if (c0 + off < V) x = *reinterpret_cast<const float4 *>(stage + off);
+            if (inside || off < V) x = ldg_stream4(reinterpret_cast<const float4 *>(row + off));  // V % 4 == 0
             v[4 * j + 0] = x.x;
             v[4 * j + 1] = x.y;
             v[4 * j + 2] = x.z;
@@ -163,50 +150,22 @@ __device__ __forceinline__ void read_item(const float *stage, int V, int c0, flo
     } else {
 #pragma unroll
         for (int j = 0; j < kAccVpt; ++j) {
-            const int off = j * kAccThreads + tid;
-            v[j] = c0 + off < V ? stage[off] : -INFINITY;
+            const int off = c0 + j * kAccThreads + tid;
+            v[j] = off < V ? ldg_stream(row + off) : -INFINITY;
         }
     }
-}
 
-struct RowsShared {
-    MS sms[kAccThreads / 32];
-    float thr[kAccThreads / 32];
-    VI wtop[kAccThreads / 32][RS_MAX_BETA];  // per-warp lists (tie fallback)
-    VI cbuf[kCandCap];                       // the chunk's candidates
-    int cnt;
-};
-
-// One work item on the logits in registers: the chunk's (max, sum e, sum e
-// (z - max)) triple and its best beta candidates.
-// `rw` is the warp that ranks the candidates and writes the item's results
-// (rotated over items).  `sh` alternates between two copies over items, so no
-// barrier is needed at the end: a copy is next written two items later, after
-// every thread has passed the first barrier of the item in between.
-template <bool kVec, bool kEnt>
-__device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int c0, int beta, int blk,
-                                          VI *__restrict__ cand, MS *__restrict__ part, RowsShared &sh, int rw) {
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    constexpr float kL2E = 1.4426950408889634f;
-    if (tid == 0) sh.cnt = 0;
-
-    // logit id of register j (padding slots have ids >= V)
-    auto id_of = [&](int j) -> int {
-        if (kVec) return c0 + ((j >> 2) * kAccThreads + tid) * 4 + (j & 3);
-        return c0 + j * kAccThreads + tid;
-    };
-
-    // lane maximum; the warp maximum and a lower bound on the chunk's beta-th
-    // largest logit from the sorted lane maxima: the warp holds beta lane
-    // maxima >= its beta-th largest, and each is a logit of the chunk.  Every lane exponentiates against the warp
-    // maximum, so the warp's (max, sum e, sum e (z - max)) is a plain sum.
-    float m8[8];
+    // group, lane, half-warp and warp maxima
+    float g[kAccVpt / 4];
 #pragma unroll
-    for (int q = 0; q < 8; ++q) m8[q] = fmaxf(fmaxf(v[q], v[q + 8]), fmaxf(v[q + 16], v[q + 24]));
-    const float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
-                           fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
-    float wmax, thr_w;
-    warp_max_and_bound<32>(mx, lane, beta, &wmax, &thr_w);
+    for (int q = 0; q < kAccVpt / 4; ++q) g[q] = fmaxf(fmaxf(v[4 * q], v[4 * q + 1]), fmaxf(v[4 * q + 2], v[4 * q + 3]));
+    const float mx = fmaxf(fmaxf(fmaxf(g[0], g[1]), fmaxf(g[2], g[3])), fmaxf(fmaxf(g[4], g[5]), fmaxf(g[6], g[7])));
+    float hm = mx;
+#pragma unroll
+    for (int o = 1; o < 16; o <<= 1) hm = fmaxf(hm, __shfl_xor_sync(0xffffffffu, hm, o));
+    const float wmax = fmaxf(hm, __shfl_xor_sync(0xffffffffu, hm, 16));
+    if ((lane & 15) == 0) sh.hmax[2 * warp + (lane >> 4)] = hm;
+
     MS t{wmax, 0.f, 0.f};
     if (wmax != -INFINITY) {
         // base 2: u = (z - max) log2(e), e = 2^u; sum e (z - max) = ln 2 sum e u
@@ -234,29 +193,23 @@ __device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int 
         t.s = ss;
         t.w = ww * 0.6931471805599453f;
     }
-    if (lane == 0) {
-        sh.sms[warp] = t;
-        sh.thr[warp] = thr_w;
-    }
-
-    // ---- the chunk's best beta, exactly, in (logit desc, id asc) order ----
-    // Only logits >= T = max over warps of the bounds can be in the chunk's
-    // best beta; they are appended to one shared buffer and ranked by one
-    // warp (each candidate's rank = the number of candidates before it).  If
-    // ties overflow the buffer, every warp ranks its own logits and that warp
-    // merges the eight lists instead.
+    if (lane == 0) sh.sms[warp] = t;
     __syncthreads();
-    float thr = sh.thr[0];
-#pragma unroll
-    for (int w = 1; w < kAccThreads / 32; ++w) thr = fmaxf(thr, sh.thr[w]);
+
+    // T = the beta-th largest half-warp maximum (both half-warps sort the same 16)
+    const float thr = __shfl_sync(0xffffffffu, group_sort_desc<16>(sh.hmax[lane & 15], lane), beta - 1);
     if (mx >= thr) {
 #pragma unroll
-        for (int j = 0; j < kAccVpt; ++j) {
-            if (v[j] >= thr) {
-                const int id = id_of(j);
-                if (id < V) {
-                    const int p = atomicAdd(&sh.cnt, 1);
-                    if (p < kCandCap) sh.cbuf[p] = VI{v[j], id};
+        for (int q = 0; q < kAccVpt / 4; ++q) {
+            if (g[q] >= thr) {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int j = 4 * q + e;
+                    const int id = id_of(j);
+                    if (v[j] >= thr && id < V) {
+                        const int p = atomicAdd(&sh.cnt, 1);
+                        if (p < kCandCap) sh.cbuf[p] = VI{v[j], id};
+                    }
                 }
             }
         }
@@ -264,7 +217,7 @@ __device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int 
     __syncthreads();
     const int total = sh.cnt;
     if (total <= kCandCap) {
-        if (warp == rw) {
+        if (warp == 0) {
             VI x0 = lane < total ? sh.cbuf[lane] : VI{-INFINITY, kNoId};
             VI x1 = lane + 32 < total ? sh.cbuf[lane + 32] : VI{-INFINITY, kNoId};
             int r0 = 0, r1 = 0;
@@ -273,9 +226,9 @@ __device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int 
                 r0 += vi_before(y.v, y.i, x0.v, x0.i);
                 r1 += vi_before(y.v, y.i, x1.v, x1.i);
             }
-            if (lane < total && r0 < beta) cand[(long long)blk * beta + r0] = x0;
-            if (lane + 32 < total && r1 < beta) cand[(long long)blk * beta + r1] = x1;
-            if (lane >= total && lane < beta) cand[(long long)blk * beta + lane] = VI{-INFINITY, kNoId};
+            if (lane < total && r0 < beta) cand[blk * beta + r0] = x0;
+            if (lane + 32 < total && r1 < beta) cand[blk * beta + r1] = x1;
+            if (lane >= total && lane < beta) cand[blk * beta + lane] = VI{-INFINITY, kNoId};
         }
     } else {
         VI prev{INFINITY, -1};
@@ -292,7 +245,7 @@ __device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int 
             if (lane == 0) sh.wtop[warp][k] = best;
         }
         __syncthreads();
-        if (warp == rw) {
+        if (warp == 0) {
             constexpr int kW = kAccThreads / 32;
             VI prevb{INFINITY, -1};
             for (int k = 0; k < beta; ++k) {
@@ -305,44 +258,15 @@ __device__ __forceinline__ void rows_item(const float (&v)[kAccVpt], int V, int 
                 }
                 best = warp_vi_best(best);
                 prevb = best;
-                if (lane == 0) cand[(long long)blk * beta + k] = best;
+                if (lane == 0) cand[blk * beta + k] = best;
             }
         }
     }
-    if (warp == rw) {  // the eight warp triples, merged as a 3-level tree
+    if (warp == 0) {  // the eight warp triples, merged as a 3-level tree
         MS a = lane < kAccThreads / 32 ? sh.sms[lane] : MS{-INFINITY, 0.f, 0.f};
 #pragma unroll
         for (int o = 4; o > 0; o >>= 1) a = ms_merge(a, ms_shfl(a, o));
         if (lane == 0) part[blk] = a;
-    }
-}
-
-// Persistent over work items: while a CTA works on item i, the copies of
-// item i + gridDim.x into the other shared-memory stage are in flight.
-constexpr int kRowsStages = 2;
-constexpr size_t kRowsSmem = (size_t)kRowsStages * kAccChunk * sizeof(float);
-
-template <bool kVec, bool kEnt>
-__global__ void __launch_bounds__(kAccThreads, 3)
-accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, int n_items,
-            VI *__restrict__ cand, MS *__restrict__ part) {
-    pdl_enter();
-    __shared__ RowsShared sh[2];
-    extern __shared__ __align__(16) float s_stage[];  // kRowsStages x kAccChunk
-    const int step = gridDim.x;
-    int item = blockIdx.x;
-    if (item < n_items) fetch_item<kVec>(logits, V, nchunks, item, s_stage);
-    cp_async_commit();
-    for (int k = 0; item < n_items; ++k, item += step) {
-        float *cur = s_stage + (k & 1) * kAccChunk;
-        float *nxt = s_stage + ((k + 1) & 1) * kAccChunk;
-        if (item < n_items - step) fetch_item<kVec>(logits, V, nchunks, item + step, nxt);
-        cp_async_commit();
-        cp_async_wait_1();  // this thread's copies of `item` have landed
-        const int c0 = (item % nchunks) * kAccChunk;
-        float v[kAccVpt];
-        read_item<kVec>(cur, V, c0, v);
-        rows_item<kVec, kEnt>(v, V, c0, beta, item, cand, part, sh[k & 1], k % (kAccThreads / 32));
     }
 }
 
@@ -730,42 +654,18 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
     if (R > 0) {
         const long long blocks = (long long)R * nchunks;
         RS_CHECK_ARG(blocks < (1ll << 30), "rs_accept: R*chunks too large");
-        const int n_items = (int)blocks;
         const bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
         const bool ent = entropy != nullptr;
-        const unsigned grid = (unsigned)std::min<long long>(blocks, 3ll * num_sms());
-        static int attr_done[64] = {0};
-        int dev = 0;
-        cudaGetDevice(&dev);
-        if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-            cudaError_t e = cudaSuccess;
-            const int bytes = (int)kRowsSmem;
-            if (e == cudaSuccess)
-                e = cudaFuncSetAttribute(accept_rows<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-            if (e == cudaSuccess)
-                e = cudaFuncSetAttribute(accept_rows<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-            if (e == cudaSuccess)
-                e = cudaFuncSetAttribute(accept_rows<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-            if (e == cudaSuccess)
-                e = cudaFuncSetAttribute(accept_rows<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-            if (e != cudaSuccess) {
-                set_error("rs_accept: cudaFuncSetAttribute: %s", cudaGetErrorString(e));
-                return RS_ERR_CUDA;
-            }
-            attr_done[dev] = 1;
-        }
+        const dim3 grid((unsigned)blocks);
         if (vec && ent)
-            launch_full(accept_rows<true, true>, dim3(grid), dim3(kAccThreads), kRowsSmem, st, logits, V, nchunks,
-                p.beta, n_items, cand, part);
+            launch_pdl(accept_rows<true, true>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand, part);
         else if (vec)
-            launch_full(accept_rows<true, false>, dim3(grid), dim3(kAccThreads), kRowsSmem, st, logits, V,
-                nchunks, p.beta, n_items, cand, part);
+            launch_pdl(accept_rows<true, false>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand, part);
         else if (ent)
-            launch_full(accept_rows<false, true>, dim3(grid), dim3(kAccThreads), kRowsSmem, st, logits, V,
-                nchunks, p.beta, n_items, cand, part);
+            launch_pdl(accept_rows<false, true>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand, part);
         else
-            launch_full(accept_rows<false, false>, dim3(grid), dim3(kAccThreads), kRowsSmem, st, logits, V,
-                nchunks, p.beta, n_items, cand, part);
+            launch_pdl(accept_rows<false, false>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand,
+                part);
         RS_CHECK_LAUNCH("rs_accept/accept_rows");
         launch_pdl(accept_merge, dim3((R + kMergeThreads / 32 - 1) / (kMergeThreads / 32)), dim3(kMergeThreads),
             0, st, cand, part, nchunks, p.beta, R, argmax, topk, lse, entropy, rowmax);
