@@ -122,7 +122,7 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
     pdl_enter();
     __shared__ RowsShared sh;
     const long long blk = blockIdx.x;
-    const long long r = blk / nchunks;
+    const long long r = blockIdx.x / (unsigned)nchunks;  // 32-bit division
     const int c0 = (int)(blk - r * nchunks) * kAccChunk;
     const float *row = logits + r * (long long)V;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;

@@ -60,7 +60,7 @@ __global__ void __launch_bounds__(kGateThreads)
 entropy_partial(const float *__restrict__ logits, int V, int nchunks, Ent3 *__restrict__ part) {
     pdl_enter();
     const long long blk = blockIdx.x;
-    const long long r = blk / nchunks;
+    const long long r = blockIdx.x / (unsigned)nchunks;  // 32-bit division
     const int chunk = (int)(blk - r * nchunks);
     const float *row = logits + r * (long long)V;
     const int c0 = chunk * kGateChunk;

@@ -9,7 +9,8 @@
 // token-id order, of a caller-supplied uniform u:  the smallest id v with
 // sum_{w <= v} p_T(w) > u.
 //
-// Kernel 1 (sample_partial): one CTA per (row, 8192-logit chunk); thread t
+// Kernel 1 (sample_partial): one CTA per (row, 8192-logit chunk), staged
+// through shared memory with coalesced loads; thread t
 // owns the 32 consecutive ids c0 + 32 t .. c0 + 32 t + 31 and sums
 // e_v = 2^((z_v - m_c) log2(e) / T) over them in id order, m_c being the
 // chunk maximum; the chunk's (m_c, s_c) go to the workspace.
@@ -64,6 +65,40 @@ __device__ __forceinline__ void load32(const float *__restrict__ row, int V, int
     }
 }
 
+// The same 32 logits, read through shared memory: the CTA streams the chunk
+// with coalesced 128-bit loads into a buffer padded by four floats after
+// every 32 (so that neither the stores nor the per-thread 128-bit reads of 32
+// consecutive ids meet bank conflicts), then each thread takes its own ids.
+// Chunks that end past V fall back to load32.  The values are the same either
+// way, so the per-thread sums do not depend on the path.
+constexpr int kSmpPadded = kSmpChunk + kSmpChunk / 8;  // 36 floats per thread
+
+template <bool kVec>
+__device__ __forceinline__ void load32_staged(const float *__restrict__ row, int V, int c0, float *s_buf,
+                                              float (&z)[kSmpVpt]) {
+    if (kVec && c0 + kSmpChunk <= V) {  // uniform over the CTA
+        const int tid = threadIdx.x;
+#pragma unroll
+        for (int j = 0; j < kSmpVpt / 4; ++j) {
+            const int e = 4 * (j * kSmpThreads + tid);
+            const float4 x = ldg_stream4(reinterpret_cast<const float4 *>(row + c0 + e));
+            *reinterpret_cast<float4 *>(s_buf + e + 4 * (e >> 5)) = x;
+        }
+        __syncthreads();
+        const float4 *p = reinterpret_cast<const float4 *>(s_buf + tid * (kSmpVpt + 4));
+#pragma unroll
+        for (int q = 0; q < kSmpVpt / 4; ++q) {
+            const float4 x = p[q];
+            z[4 * q] = x.x;
+            z[4 * q + 1] = x.y;
+            z[4 * q + 2] = x.z;
+            z[4 * q + 3] = x.w;
+        }
+    } else {
+        load32<kVec>(row, V, c0, z);
+    }
+}
+
 __device__ __forceinline__ float block_max(float v, float *s_w) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     v = warp_max(v);
@@ -104,10 +139,11 @@ __global__ void __launch_bounds__(kSmpThreads)
 sample_partial(const float *__restrict__ logits, int V, int nchunks, float scale, ChunkMass *__restrict__ part) {
     pdl_enter();
     __shared__ float s_w[kSmpThreads / 32];
+    __shared__ __align__(16) float s_buf[kSmpPadded];
     const int r = blockIdx.x / nchunks, c = blockIdx.x - r * nchunks;
     const float *row = logits + (long long)r * V;
     float z[kSmpVpt];
-    load32<kVec>(row, V, c * kSmpChunk, z);
+    load32_staged<kVec>(row, V, c * kSmpChunk, s_buf, z);
     float mx = -INFINITY;
 #pragma unroll
     for (int j = 0; j < kSmpVpt; ++j) mx = fmaxf(mx, z[j]);
@@ -132,6 +168,7 @@ sample_pick(const float *__restrict__ logits, int V, int nchunks, float scale, c
     __shared__ int s_chunk;
     __shared__ float s_target;  // u Z within the chosen chunk, in its own units
     __shared__ int s_draw;
+    __shared__ __align__(16) float s_buf[kSmpPadded];
     const int r = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31;
     const ChunkMass *pr = part + (long long)r * nchunks;
@@ -199,7 +236,7 @@ sample_pick(const float *__restrict__ logits, int V, int nchunks, float scale, c
     const float nb = -m * scale;
     const float *row = logits + (long long)r * V;
     float z[kSmpVpt];
-    load32<kVec>(row, V, c * kSmpChunk, z);
+    load32_staged<kVec>(row, V, c * kSmpChunk, s_buf, z);
     float s = 0.f;
 #pragma unroll
     for (int j = 0; j < kSmpVpt; ++j) s += ex2f(fmaf(z[j], scale, nb));
