@@ -16,7 +16,7 @@
 //   attn_prep validates each tree and builds a 256-bit ancestor set per
 //   node; the tree part of the mask is a bit test on it.
 // Launches: attn_prep (B CTAs) -> attn_tc_kernel (one CTA per SM; see
-// attn_core.cuh) -> attn_combine (four CTAs per range).
+// attn_core.cuh) -> attn_combine (three CTAs per SM over the split segments' rows).
 #include <cudaTypedefs.h>
 #include <math.h>
 
@@ -83,159 +83,160 @@ attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_
     if (tid == 0) status[b] = st;
 }
 
-// Block (c, y) merges rows [32 y, 32 y + 32) of the split segment CTA c of
-// the attention kernel started (its job record; four blocks per segment).
-// The segment's pieces are the partials of CTA c (slot first_slot) and of
-// slot 0 of every later CTA up to c1 with a non-empty range.
-// Phase 1: thread (row r, lane group j) folds the (m, l) pairs of pieces j,
-// j + 8, ... into a running (max, sum); warp 0 merges the eight folds into the
-// row's M = max_p m_p and 1 / L, L = sum_p e^(m_p - M) l_p.  Phase 2: each
-// thread owns D / 32 (row, 4 head-dim columns) items and sums e^(m_p - M) O_p
-// over the pieces, two pieces per round, so a round keeps 2 x D / 32 float4
-// partial loads and their m_p loads in flight (the first round is issued
-// before phase 1, so the two phases share one memory round trip).  The
-// summation order is fixed (piece order), so the result does not depend on
-// timing.
+// attn_combine: every block first reads all job records (one per attention
+// CTA; a record names the split segment that CTA started) and cuts each job
+// into items of rows by a block scan, then takes items blockIdx.x,
+// blockIdx.x + gridDim.x, ...  A lane merges one column quad of rpw
+// consecutive rows, rpw = 4, 2 or 1 for segments of <= 2, <= 4 or more
+// pieces, so that it issues the loads of up to kCombPairs (row, piece)
+// partials (o, m, l) at once: an item costs one memory round trip for
+// segments of up to eight pieces whatever their number.  The pieces of a
+// row are folded in piece order with a running maximum (deterministic):
+// M = max_p m_p, L = sum_p e^(m_p - M) l_p, O = sum_p e^(m_p - M) O_p / L.
+// The pieces of a segment are the partial of CTA c (slot first_slot) and
+// slot 0 of every later CTA up to c1 with a non-empty range: with at least
+// as many units as CTAs every range is non-empty, otherwise every non-empty
+// range holds one unit.
 constexpr int kCombThreads = 256;
-constexpr int kCombRows = 32;                    // rows per block
-constexpr int kCombGroups = kBM / kCombRows;     // blocks per split segment
-constexpr int kCombFold = kCombThreads / kCombRows;  // lane groups in phase 1
-constexpr int kCombBatch = 2;                    // pieces per phase-2 round
+constexpr int kCombPairs = 8;  // (row, piece) loads in flight per lane
 
-__global__ void __launch_bounds__(kCombThreads, 4)  // the 4 x Gc blocks in one wave
-attn_combine(AttnArgs a) {
-    pdl_enter();
-    __shared__ int s_slot[kAttnMaxGrid];
-    __shared__ float s_fm[kCombFold][kCombRows], s_fl[kCombFold][kCombRows];
-    __shared__ float s_M[kCombRows], s_iL[kCombRows];
-    const int c = blockIdx.x;
-    const CombJob job = a.jobs[c];
-    if (job.b < 0) return;
+__device__ __forceinline__ int comb_np(const CombJob &j, int c, long long Gc) {
+    return j.W >= Gc ? j.c1 - c + 1 : (int)(range_lo(j.c1 + 1, j.W, Gc) - range_lo(c, j.W, Gc));
+}
+
+template <int D>
+__device__ __forceinline__ void combine_item(const AttnArgs &a, const CombJob &job, int c, int np, long long Gc,
+                                             int row0, int rpw) {
+    constexpr int kLpr = D / 4;        // lanes per row, one column quad each
+    constexpr int kSub = 32 / kLpr;    // row groups per warp
+    const int lane = threadIdx.x & 31;
+    const int q = lane % kLpr;
+    const int grp = (int)(threadIdx.x >> 5) * kSub + lane / kLpr;
     const int G = a.Hq / a.Hkv;
-    const int n0 = job.n0, N = job.N, kvh = job.kvh, mtile = job.mtile;
-    const int r0 = blockIdx.y * kCombRows;
-    const int rows = min(kCombRows, N * G - mtile * kBM - r0);
-    if (rows <= 0) return;
-    const long long Gc = gridDim.x;
-    int np;
-    if (job.W >= Gc) {  // every range is non-empty: one piece per CTA c .. c1
-        np = job.c1 - c + 1;
-        for (int x = threadIdx.x; x < np; x += kCombThreads) s_slot[x] = x == 0 ? job.first_slot : 2 * (c + x);
-    } else {
-        __shared__ int s_np;
-        if (threadIdx.x == 0) {
-            int n = 0;
-            s_slot[n++] = job.first_slot;
-            for (long long cc = c + 1; cc <= job.c1 && n < kAttnMaxGrid; ++cc)
-                if (range_lo(cc, job.W, Gc) < range_lo(cc + 1, job.W, Gc)) s_slot[n++] = (int)(2 * cc);
-            s_np = n;
-        }
-        __syncthreads();
-        np = s_np;
-    }
-    __syncthreads();
-    const int D = a.D;
-
-    // phase-2 items of this thread (row, column quad), and the first batch of
-    // their partial loads, issued before phase 1 so both share one round trip
-    constexpr int kMaxItems = kCombRows * 128 / 4 / kCombThreads;  // 4 for D = 128
-    const int d4 = D / 4;
-    const int nitems = rows * d4;
-    float4 acc[kMaxItems];
-    int irow[kMaxItems];
-#pragma unroll
-    for (int k = 0; k < kMaxItems; ++k) {
-        acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-        const int x = threadIdx.x + k * kCombThreads;
-        irow[k] = x < nitems ? x / d4 : -1;
-    }
-    float m[kCombBatch][kMaxItems];
-    float4 o[kCombBatch][kMaxItems];
-    auto load_batch = [&](int p0) {
-#pragma unroll
-        for (int q = 0; q < kCombBatch; ++q) {
-            const long long base = p0 + q < np ? (long long)s_slot[p0 + q] * kBM + r0 : -1;
-#pragma unroll
-            for (int k = 0; k < kMaxItems; ++k) {
-                m[q][k] = -INFINITY;
-                o[q][k] = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (base >= 0 && irow[k] >= 0) {
-                    const int x = threadIdx.x + k * kCombThreads;
-                    const int r = irow[k], cq = x - r * d4;
-                    m[q][k] = a.part_m[base + r];
-                    o[q][k] = *reinterpret_cast<const float4 *>(a.part_o + (base + r) * D + cq * 4);
-                }
-            }
-        }
+    const int rows = min(kBM, job.N * G - job.mtile * kBM);
+    const int rbase = row0 + grp * rpw;                 // this lane's first row in the tile
+    const int npairs = max(0, min(rpw, rows - rbase)) * np;
+    const bool fast = job.W >= Gc;
+    const long long u_c = fast ? 0 : range_lo(c, job.W, Gc);
+    auto slot_of = [&](int p) -> long long {
+        if (p == 0) return job.first_slot;
+        return fast ? 2ll * (c + p) : 2ll * owner_of(u_c + p, job.W, Gc);
     };
-    load_batch(0);
-
-    // phase 1: per-row M and 1 / L
-    {
-        const int r = threadIdx.x & (kCombRows - 1), j = threadIdx.x / kCombRows;
-        float fm = -INFINITY, fl = 0.f;
-        if (r < rows) {
-            for (int p = j; p < np; p += kCombFold) {
-                const long long prow = (long long)s_slot[p] * kBM + r0 + r;
-                const float mp = a.part_m[prow], lp = a.part_l[prow];
-                if (mp == -INFINITY) continue;
-                if (mp > fm) {
-                    fl = fl * __expf(fm - mp) + lp;  // fm = -inf: fl = 0
-                    fm = mp;
-                } else {
-                    fl += lp * __expf(mp - fm);
+    float M = -INFINITY, L = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    int k = 0, p = 0;  // row and piece the fold is at
+    for (int x0 = 0; x0 < npairs; x0 += kCombPairs) {
+        float m[kCombPairs], l[kCombPairs];
+        float4 o[kCombPairs];
+        {
+            int kk = x0 / np, pp = x0 - kk * np;
+#pragma unroll
+            for (int s = 0; s < kCombPairs; ++s) {
+                m[s] = -INFINITY;
+                l[s] = 0.f;
+                o[s] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (x0 + s < npairs) {
+                    const long long prow = slot_of(pp) * kBM + rbase + kk;
+                    m[s] = a.part_m[prow];
+                    l[s] = a.part_l[prow];
+                    o[s] = *reinterpret_cast<const float4 *>(a.part_o + prow * D + q * 4);
+                    if (++pp == np) {
+                        pp = 0;
+                        ++kk;
+                    }
                 }
             }
         }
-        s_fm[j][r] = fm;
-        s_fl[j][r] = fl;
-        __syncthreads();
-        if (threadIdx.x < kCombRows) {
-            float M = -INFINITY;
 #pragma unroll
-            for (int q = 0; q < kCombFold; ++q) M = fmaxf(M, s_fm[q][r]);
-            float L = 0.f;
-#pragma unroll
-            for (int q = 0; q < kCombFold; ++q)
-                if (s_fm[q][r] != -INFINITY) L += s_fl[q][r] * __expf(s_fm[q][r] - M);
-            s_M[r] = M;
-            s_iL[r] = L > 0.f ? 1.f / L : 0.f;
-            if (r < rows) {
-                const int rr = mtile * kBM + r0 + r;
-                const int i = rr / G, h = kvh * G + (rr - i * G);
-                a.lse[(long long)(n0 + i) * a.Hq + h] = M + __logf(L);
+        for (int s = 0; s < kCombPairs; ++s) {
+            if (x0 + s >= npairs) break;
+            const float mp = m[s];
+            if (mp != -INFINITY) {
+                if (mp > M) {
+                    const float sc = __expf(M - mp);  // M = -inf: 0
+                    acc = make_float4(fmaf(acc.x, sc, o[s].x), fmaf(acc.y, sc, o[s].y), fmaf(acc.z, sc, o[s].z),
+                                      fmaf(acc.w, sc, o[s].w));
+                    L = fmaf(L, sc, l[s]);
+                    M = mp;
+                } else {
+                    const float w = __expf(mp - M);
+                    acc = make_float4(fmaf(w, o[s].x, acc.x), fmaf(w, o[s].y, acc.y), fmaf(w, o[s].z, acc.z),
+                                      fmaf(w, o[s].w, acc.w));
+                    L = fmaf(w, l[s], L);
+                }
+            }
+            if (++p == np) {  // row rbase + k complete
+                const int rr = job.mtile * kBM + rbase + k;
+                const int i = rr / G, h = job.kvh * G + (rr - i * G);
+                const long long orow = (long long)(job.n0 + i) * a.Hq + h;
+                const float f = L > 0.f ? 1.f / L : 0.f;
+                *reinterpret_cast<float4 *>(a.out + orow * D + q * 4) =
+                    make_float4(acc.x * f, acc.y * f, acc.z * f, acc.w * f);
+                if (q == 0) a.lse[orow] = M + __logf(L);
+                M = -INFINITY;
+                L = 0.f;
+                acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                p = 0;
+                ++k;
             }
         }
-        __syncthreads();
     }
+}
 
-    // phase 2: the weighted sum of the partial outputs, kCombBatch pieces a round
-    for (int p0 = 0; p0 < np; p0 += kCombBatch) {
-        if (p0 > 0) load_batch(p0);
-#pragma unroll
-        for (int q = 0; q < kCombBatch; ++q) {
-#pragma unroll
-            for (int k = 0; k < kMaxItems; ++k) {
-                if (irow[k] < 0 || m[q][k] == -INFINITY) continue;
-                const float w = __expf(m[q][k] - s_M[irow[k]]);
-                acc[k].x = fmaf(w, o[q][k].x, acc[k].x);
-                acc[k].y = fmaf(w, o[q][k].y, acc[k].y);
-                acc[k].z = fmaf(w, o[q][k].z, acc[k].z);
-                acc[k].w = fmaf(w, o[q][k].w, acc[k].w);
-            }
+template <int D>
+__global__ void __launch_bounds__(kCombThreads, 3)
+attn_combine(AttnArgs a, int Gc) {
+    pdl_enter();
+    __shared__ CombJob s_job[kAttnMaxGrid];
+    __shared__ int s_np[kAttnMaxGrid], s_rpw[kAttnMaxGrid];
+    __shared__ int s_pre[kAttnMaxGrid + 1];
+    __shared__ int s_w[kCombThreads / 32];
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int G = a.Hq / a.Hkv;
+    constexpr int rows_per_group = kCombThreads / (D / 4);  // rows of an item with rpw = 1
+    // items of the job of CTA t
+    int items = 0;
+    if (t < Gc) {
+        const CombJob j = a.jobs[t];
+        s_job[t] = j;
+        if (j.b >= 0) {
+            const int np = comb_np(j, t, Gc);
+            const int rpw = np <= 2 ? 4 : (np <= 4 ? 2 : 1);
+            const int rows = min(kBM, j.N * G - j.mtile * kBM);
+            const int per = rows_per_group * rpw;
+            s_np[t] = np;
+            s_rpw[t] = rpw;
+            items = (rows + per - 1) / per;
         }
     }
+    // exclusive prefix of the item counts (CTA order)
+    int x = items;
 #pragma unroll
-    for (int k = 0; k < kMaxItems; ++k) {
-        if (irow[k] < 0) continue;
-        const int x = threadIdx.x + k * kCombThreads;
-        const int r = irow[k], cq = x - r * d4;
-        const int rr = mtile * kBM + r0 + r;
-        const int i = rr / G, h = kvh * G + (rr - i * G);
-        const long long orow = (long long)(n0 + i) * a.Hq + h;
-        const float f = s_iL[r];
-        *reinterpret_cast<float4 *>(a.out + orow * D + cq * 4) =
-            make_float4(acc[k].x * f, acc[k].y * f, acc[k].z * f, acc[k].w * f);
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) s_w[warp] = x;
+    __syncthreads();
+    int before = 0, total = 0;
+#pragma unroll
+    for (int w = 0; w < kCombThreads / 32; ++w) {
+        before += w < warp ? s_w[w] : 0;
+        total += s_w[w];
+    }
+    if (t < Gc) s_pre[t] = before + x - items;
+    if (t == 0) s_pre[Gc] = total;
+    __syncthreads();
+    for (int it = blockIdx.x; it < total; it += gridDim.x) {
+        int lo = 0, hi = Gc - 1;  // last CTA c with s_pre[c] <= it
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (s_pre[mid] <= it) lo = mid;
+            else hi = mid - 1;
+        }
+        const int c = lo;
+        const int row0 = (it - s_pre[c]) * rows_per_group * s_rpw[c];
+        combine_item<D>(a, s_job[c], c, s_np[c], Gc, row0, s_rpw[c]);
     }
 }
 
@@ -378,7 +379,10 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     else
         launch_full(attn_tc_kernel<64>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/main");
-    launch_pdl(attn_combine, dim3(Gc, kCombGroups), dim3(kCombThreads), 0, st, a);
+    // a full launch: combine blocks parked early beside the attention CTAs
+    // (programmatic launch) measured slower on the batched workload
+    if (D == 128) launch_full(attn_combine<128>, dim3(3 * Gc), dim3(kCombThreads), 0, st, a, Gc);
+    else launch_full(attn_combine<64>, dim3(3 * Gc), dim3(kCombThreads), 0, st, a, Gc);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/combine");
     return RS_OK;
 }

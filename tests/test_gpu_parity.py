@@ -50,6 +50,10 @@ SMALL = [
          max_depth=12, n_chains=(1, 3), chain_len=12, tau=0.5, m=1, phi=3),
     dict(seed=6, B=7, Hq=8, Hkv=1, D=128, V=512, ctx=(5, 400), model_nodes=(1, 6), n_chains=(0, 1),
          chain_len=3, repeat_prob=0.6, seg_len=(2, 6), score_noise=0.6, theta_score=0.45),
+    # D = 64 with two or three 128-row tiles per KV head and enough KV tiles
+    # that every CTA's range is non-empty: split segments of several pieces
+    dict(seed=7, B=3, Hq=8, Hkv=4, D=64, V=2048, ctx=(1500, 2500), model_nodes=(80, 120), max_depth=8,
+         n_chains=(1, 3), chain_len=8),
 ]
 
 
