@@ -460,13 +460,18 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                 tc_fence_after();
                 const uint32_t s_tm = tmem + lane_off + kTmS + (uint32_t)buf * 128;
                 float s[64];
-#pragma unroll
-                for (int ch = 0; ch < 2; ++ch) {
-                    uint32_t x[32];
-                    tmem_ld32(s_tm + hw * 64 + ch * 32, x);
+                {  // both halves in flight, one wait
+                    uint32_t xa[32], xb[32];
+                    tmem_ld32(s_tm + hw * 64, xa);
+                    tmem_ld32(s_tm + hw * 64 + 32, xb);
                     tmem_wait_ld();
+                    tmem_regs_ready(xa);
+                    tmem_regs_ready(xb);
 #pragma unroll
-                    for (int e = 0; e < 32; ++e) s[ch * 32 + e] = __uint_as_float(x[e]);
+                    for (int e = 0; e < 32; ++e) {
+                        s[e] = __uint_as_float(xa[e]);
+                        s[32 + e] = __uint_as_float(xb[e]);
+                    }
                 }
                 // raw-score maximum over this half's visible keys
                 float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
@@ -547,19 +552,23 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
             const long long orow = (long long)(n0 + i) * a.Hq + h;
             const long long prow = (long long)pc.slot * kBM + r;
             const float f = pc.final ? ((lt > 0.f) ? 1.f / lt : 0.f) : 1.f;
+            uint32_t xo[kHalfO / 32][32];  // this half of O, all chunks in flight, one wait
+#pragma unroll
+            for (int ch = 0; ch < kHalfO / 32; ++ch) tmem_ld32(tmem + lane_off + kTmO + hw * kHalfO + ch * 32, xo[ch]);
+            tmem_wait_ld();
+#pragma unroll
+            for (int ch = 0; ch < kHalfO / 32; ++ch) tmem_regs_ready(xo[ch]);
 #pragma unroll
             for (int ch = 0; ch < kHalfO / 32; ++ch) {
-                uint32_t x[32];
                 const int col = hw * kHalfO + ch * 32;
-                tmem_ld32(tmem + lane_off + kTmO + col, x);
-                tmem_wait_ld();
                 if (valid) {
                     float4 *dst = pc.final ? reinterpret_cast<float4 *>(a.out + orow * D + col)
                                            : reinterpret_cast<float4 *>(a.part_o + prow * D + col);
 #pragma unroll
                     for (int e = 0; e < 8; ++e)
-                        dst[e] = make_float4(__uint_as_float(x[4 * e]) * f, __uint_as_float(x[4 * e + 1]) * f,
-                                             __uint_as_float(x[4 * e + 2]) * f, __uint_as_float(x[4 * e + 3]) * f);
+                        dst[e] = make_float4(__uint_as_float(xo[ch][4 * e]) * f, __uint_as_float(xo[ch][4 * e + 1]) * f,
+                                             __uint_as_float(xo[ch][4 * e + 2]) * f,
+                                             __uint_as_float(xo[ch][4 * e + 3]) * f);
                 }
             }
             if (valid && hw == 0) {

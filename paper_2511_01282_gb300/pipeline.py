@@ -31,7 +31,7 @@ class VerifyStep:
               "chain", "sel_pos")
 
     def __init__(self, arrays, p, Hq, Hkv, D, pos_cap=1024, acc_cap=64, device="cuda",
-                 scale=None, pinned_host=False, sample_seed=0):
+                 scale=None, pinned_host=False, sample_seed=0, host_blob=None):
         self.p = p
         self.Hq, self.Hkv, self.D = Hq, Hkv, D
         self.scale = float(D ** -0.5 if scale is None else scale)
@@ -44,11 +44,31 @@ class VerifyStep:
         self.R = int(self.host["node_off"][-1])
         self.V = int(self.host["logits"].shape[1])
         self.kv_rows = int(self.host["k"].shape[0])
-        # device inputs
-        self.d = {k: _dev(v, self.device) for k, v in self.host.items()}
-        self.pinned = None
-        if pinned_host:
-            self.pinned = {k: torch.from_numpy(v).pin_memory() for k, v in self.host.items()}
+        # device inputs.  With pinned_host the inputs live in one device
+        # allocation (256-byte aligned views) mirrored by one pinned host
+        # buffer, so that a step's upload is a single copy; host_blob shares
+        # another VerifyStep's pinned buffer (same arrays).
+        self.pinned_blob = None
+        if pinned_host or host_blob is not None:
+            layout, off = {}, 0
+            for k, v in self.host.items():
+                layout[k] = (off, v.nbytes, v.dtype, v.shape)
+                off += -(-max(v.nbytes, 1) // 256) * 256
+            if host_blob is None:
+                host_blob = torch.empty(off, dtype=torch.uint8).pin_memory()
+                hb = host_blob.numpy()
+                for k, v in self.host.items():
+                    o, n = layout[k][:2]
+                    hb[o:o + n] = v.reshape(-1).view(np.uint8)
+            assert host_blob.numel() == off and host_blob.is_pinned()
+            self.pinned_blob = host_blob
+            self.dev_blob = torch.empty(off, dtype=torch.uint8, device=self.device)
+            self.dev_blob.copy_(host_blob)
+            tdt = lambda dt: torch.from_numpy(np.empty(0, dt)).dtype  # noqa: E731  (as torch.from_numpy maps it)
+            self.d = {k: self.dev_blob[o:o + n].view(tdt(dt)).reshape(shape)
+                      for k, (o, n, dt, shape) in layout.items()}
+        else:
+            self.d = {k: _dev(v, self.device) for k, v in self.host.items()}
         B, R, V = self.B, self.R, self.V
         dev = self.device
         z = lambda n, dt: torch.zeros(n, dtype=dt, device=dev)  # noqa: E731
@@ -163,12 +183,11 @@ class VerifyStep:
 
     # ------------------------------------------------------ host round trip
     def upload(self, stream=None):
-        """Copy every input from pinned host memory (async on `stream`)."""
+        """Copy every input from pinned host memory: one async copy on `stream`."""
         s = torch.cuda.current_stream() if stream is None else stream
         with torch.cuda.stream(s):
-            for k, t in self.pinned.items():
-                self.d[k].copy_(t, non_blocking=True)
-        return sum(t.numel() * t.element_size() for t in self.pinned.values())
+            self.dev_blob.copy_(self.pinned_blob, non_blocking=True)
+        return self.pinned_blob.numel()
 
     RESULT_KEYS = ("acc_len", "acc_nodes", "bonus", "winner", "commit", "k_star", "entropy_ok",
                    "sel_pos", "n_sel")
