@@ -49,6 +49,8 @@ def parse():
     ap.add_argument("--cpu-budget-s", type=float, default=12.0,
                     help="seconds of oracle attention work in the CPU baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true",
+                    help="skip the end-to-end (host buffers) measurement: lean runs for profiling")
     ap.add_argument("--requests", type=int, default=0,
                     help="keep only the first N requests of the workload (small profiling cases)")
     return ap.parse_args()
@@ -173,6 +175,58 @@ def committed_traffic(workload):
     if not e or e.get("source_sha") != attn_source_sha():
         return None
     return e.get("dram_bytes_per_launch")
+
+
+# ------------------------------------------------------------------ end to end
+def end_to_end(st, st2, graph, stream, K, W, barrier):
+    """K steps from pinned host inputs to decisions on the host, through the
+    same calls.  Two device copies of the inputs (st, st2: one pinned host
+    buffer) alternate, so the upload of step i + 1 (copy engine) overlaps step
+    i's kernels; the host holds step i - 1's decisions before it enqueues
+    step i + 1.  Returns (seconds, h2d bytes per step, d2h bytes per step)."""
+    import torch
+    st2.prime()
+    torch.cuda.synchronize()
+    for _ in range(2):
+        st2.step(stream)
+    torch.cuda.synchronize()
+    graph2 = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph2, stream=stream):
+        st2.step(stream)
+    sets = [(st, graph, st.result_buffers()), (st2, graph2, st2.result_buffers())]
+    copy_stream = torch.cuda.Stream()
+
+    def e2e_step(i, done):
+        x = i & 1
+        sx, gx, bx = sets[x]
+        if done[x] is not None:  # step i - 2 has finished with this input set
+            copy_stream.wait_event(done[x])
+        h = sx.upload(copy_stream)
+        up = torch.cuda.Event()
+        up.record(copy_stream)
+        stream.wait_event(up)
+        with torch.cuda.stream(stream):
+            gx.replay()
+        d = sx.download_into(bx, stream)
+        ev = torch.cuda.Event()
+        ev.record(stream)
+        done[x] = ev
+        if i >= 1:  # step i - 1's decisions are on the host
+            done[x ^ 1].synchronize()
+        return h, d
+
+    done = [None, None]
+    for i in range(max(W, 2)):
+        e2e_step(i, done)
+    torch.cuda.synchronize()
+    barrier()
+    done = [None, None]
+    t0 = time.perf_counter()
+    h2d = d2h = 0
+    for i in range(K):
+        h2d, d2h = e2e_step(i, done)
+    torch.cuda.synchronize()
+    return time.perf_counter() - t0, h2d, d2h
 
 
 # ------------------------------------------------------------------ CPU oracle sample
@@ -345,55 +399,14 @@ def run_ours(args, rank, world, local_rank):
     st.reset_state()
     torch.cuda.synchronize()
 
-    # ---- end to end: pinned host inputs -> step -> decisions back to the host.
-    # Two device copies of the inputs (sharing one pinned host buffer)
-    # alternate, so the upload of step i + 1 (copy engine) overlaps step i's
-    # kernels; the host holds step i - 1's decisions before it enqueues i + 1.
-    st2 = VerifyStep(arrays_from_workload(w), p, s.Hq, s.Hkv, s.D, pos_cap=s.pos_cap, host_blob=st.pinned_blob)
-    st2.prime()
-    torch.cuda.synchronize()
-    for _ in range(2):
-        st2.step(stream)
-    torch.cuda.synchronize()
-    graph2 = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph2, stream=stream):
-        st2.step(stream)
-    sets = [(st, graph, st.result_buffers()), (st2, graph2, st2.result_buffers())]
-    copy_stream = torch.cuda.Stream()
-
-    def e2e_step(i, done):
-        x = i & 1
-        sx, gx, bx = sets[x]
-        if done[x] is not None:  # step i - 2 has finished with this input set
-            copy_stream.wait_event(done[x])
-        h = sx.upload(copy_stream)
-        up = torch.cuda.Event()
-        up.record(copy_stream)
-        stream.wait_event(up)
-        with torch.cuda.stream(stream):
-            gx.replay()
-        d = sx.download_into(bx, stream)
-        ev = torch.cuda.Event()
-        ev.record(stream)
-        done[x] = ev
-        if i >= 1:  # step i - 1's decisions are on the host
-            done[x ^ 1].synchronize()
-        return h, d
-
-    done = [None, None]
-    for i in range(max(W, 2)):
-        e2e_step(i, done)
-    torch.cuda.synchronize()
-    barrier()
-    done = [None, None]
-    t0 = time.perf_counter()
-    h2d = d2h = 0
-    for i in range(K):
-        h2d, d2h = e2e_step(i, done)
-    torch.cuda.synchronize()
-    e2e_s = time.perf_counter() - t0
-    barrier()
-    e2e_s = slowest(e2e_s, dist, "cuda")
+    # ---- end to end: pinned host inputs -> step -> decisions back to the host
+    if args.no_e2e:
+        K_e2e = 0
+    else:
+        K_e2e = K
+        st2 = VerifyStep(arrays_from_workload(w), p, s.Hq, s.Hkv, s.D, pos_cap=s.pos_cap, host_blob=st.pinned_blob)
+        e2e_s, h2d, d2h = end_to_end(st, st2, graph, stream, K, W, barrier)
+        e2e_s = slowest(e2e_s, dist, "cuda")
     clocks.stop()
 
     peaks, peak_kind = load_peaks()
@@ -421,8 +434,8 @@ def run_ours(args, rank, world, local_rank):
                      "launch_ms": call_ms["attn"], "traffic": committed_traffic(args.workload),
                      "tflops": by["flops"] / attn_s / 1e12},
         "call_ms": call_ms,
-        "e2e": {"value": job_rate(K, world, e2e_s), "unit": "steps/s", "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h},
+        "e2e": ({"value": job_rate(K, world, e2e_s), "unit": "steps/s", "h2d_bytes_per_step": h2d,
+                 "d2h_bytes_per_step": d2h} if K_e2e else None),
         "gpu_launches": launches_per_step * K,
         "launches_per_step": launches_per_step,
         "clocks": clocks.summary(),
