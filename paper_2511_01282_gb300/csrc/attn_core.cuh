@@ -228,7 +228,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                                                             ~uintptr_t(1023));
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kSmemBar);
     uint64_t *kfull = bars, *vfull = bars + kNS, *kempty = bars + 2 * kNS, *vempty = bars + 3 * kNS;
-    uint64_t *sfull = bars + 4 * kNS, *pfull = sfull + 2, *odone = pfull + 2, *qready = odone + 2;
+    uint64_t *sfull = bars + 4 * kNS, *pfull = sfull + 2, *qready = pfull + 2;
     uint64_t *ofree = qready + 1, *drain = ofree + 1;
     uint64_t *mxready = drain + 1, *lready = mxready + 2;  // softmax warpgroup exchanges
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + kSmemMisc);
@@ -247,8 +247,6 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
             mbar_init(&sfull[s], 1);
             mbar_init(&pfull[s], kSoftThreads);
         }
-        mbar_init(&odone[0], 1);
-        mbar_init(&odone[1], 1);
         mbar_init(qready, kSoftThreads);
         mbar_init(ofree, kSoftThreads);
         mbar_init(drain, 1);
@@ -386,7 +384,6 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                         umma_ts(tmem + kTmO, p_tm + ks * 8, sdesc_sw128(v_addr + ks * 2048, 16384, 1024), idO,
                                 (tl > 0 || ks > 0) ? 1u : 0u);
                     umma_commit(&vempty[st]);
-                    umma_commit(&odone[gt & 1]);
                 }
                 g += n;
                 u = pc.end;
@@ -399,11 +396,12 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
         }
     } else {
         // ---------------------------------------------------------- softmax / epilogue (rows)
-        // PV of tile t commits odone[t & 1].  Once S of tile t has been seen
-        // complete, every PV up to t - 2 is complete (S_t is issued after
-        // PV_{t-2}), so odone[b] is at most one phase behind the tile this
-        // thread asks for: a parity wait is unambiguous even though the
-        // thread waits only when it must read O (a rescale or the epilogue).
+        // P V of tile t commits vempty[t % kNS] (which also frees V's stage);
+        // the softmax waits on it when it must read O (a rescale or the
+        // epilogue).  Once S of tile t has been seen complete, every P V up to
+        // t - 2 is complete (S_t is issued after P V_{t-2}), and P V of t + 3
+        // needs this thread's own P, so the barrier has exactly the asked
+        // phase pending: the parity wait is unambiguous.
         // Warpgroup hw (0 or 1) owns keys [64 hw, 64 hw + 64) of every tile,
         // O columns [hw D/2, (hw + 1) D/2) for rescales and the epilogue, and
         // its own partial row sum; both keep the same reference maximum.
@@ -504,7 +502,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                 const float corr = grow ? ex2(m_used - mt) : 1.f;  // 0 when m_used is -inf
                 if (tl > 0 && __any_sync(0xffffffffu, grow)) {
                     const long long pv = gt - 1;  // O must hold PV of the previous tile
-                    if (!(ok = warp_wait(&odone[pv & 1], (uint32_t)((pv >> 1) & 1), s_abort))) break;
+                    if (!(ok = warp_wait(&vempty[(int)(pv % kNS)], (uint32_t)((pv / kNS) & 1), s_abort))) break;
                     tc_fence_after();
 #pragma unroll
                     for (int ch = 0; ch < kHalfO / 32; ++ch) {
@@ -546,7 +544,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
             const float lt = s_l[0][r] + s_l[1][r];
             {
                 const long long pv = g + n - 1;  // wait for PV of the last tile
-                if (!(ok = warp_wait(&odone[pv & 1], (uint32_t)((pv >> 1) & 1), s_abort))) break;
+                if (!(ok = warp_wait(&vempty[(int)(pv % kNS)], (uint32_t)((pv / kNS) & 1), s_abort))) break;
             }
             tc_fence_after();
             const long long orow = (long long)(n0 + i) * a.Hq + h;
