@@ -212,7 +212,7 @@ rs_status rs_match_scan(const int32_t *tokens, const int64_t *tok_off, int B,
  *            (j < ctx_len[b]) is row kv_off[b] + j and its tree node i is row
  *            kv_off[b] + ctx_len[b] + i.  k and v must be 16-byte aligned.
  *   kv_off   [B] int64;  ctx_len [B] int32 (>= 0);  node_off [B+1] int32;
- *            B <= 4096 requests per call; kv_rows < 2^31.
+ *            B <= 3840 requests per call; kv_rows < 2^31.
  *   parents  [R] int32 local parent index per node; parents of node 0 is -1,
  *            0 <= parents[i] < i otherwise.
  *   D in {64, 128}; Hq a multiple of Hkv (grouped-query heads h share KV

@@ -94,18 +94,36 @@ attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_
 // row are folded in piece order with a running maximum (deterministic):
 // M = max_p m_p, L = sum_p e^(m_p - M) l_p, O = sum_p e^(m_p - M) O_p / L.
 // The pieces of a segment are the partial of CTA c (slot first_slot) and
-// slot 0 of every later CTA up to c1 with a non-empty range: with at least
-// as many units as CTAs every range is non-empty, otherwise every non-empty
-// range holds one unit.
+// slot 0 of every later CTA up to c1 with a non-empty unit range (the CTAs'
+// ranges are read from the records the attention kernel leaves beside the
+// jobs, so the combine does not depend on how the work was split).
 constexpr int kCombThreads = 256;
 constexpr int kCombPairs = 8;  // (row, piece) loads in flight per lane
 
-__device__ __forceinline__ int comb_np(const CombJob &j, int c, long long Gc) {
-    return j.W >= Gc ? j.c1 - c + 1 : (int)(range_lo(j.c1 + 1, j.W, Gc) - range_lo(c, j.W, Gc));
+// Exclusive prefix of one int per thread of the block, in thread order.
+__device__ __forceinline__ int block_excl_scan(int v, int *s_w, int *total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) s_w[warp] = x;
+    __syncthreads();
+    int before = 0, sum = 0;
+#pragma unroll
+    for (int w = 0; w < kCombThreads / 32; ++w) {
+        before += w < warp ? s_w[w] : 0;
+        sum += s_w[w];
+    }
+    __syncthreads();
+    *total = sum;
+    return before + x - v;
 }
 
 template <int D>
-__device__ __forceinline__ void combine_item(const AttnArgs &a, const CombJob &job, int c, int np, long long Gc,
+__device__ __forceinline__ void combine_item(const AttnArgs &a, const CombJob &job, int np, const int *nonempty,
                                              int row0, int rpw) {
     constexpr int kLpr = D / 4;        // lanes per row, one column quad each
     constexpr int kSub = 32 / kLpr;    // row groups per warp
@@ -116,12 +134,8 @@ __device__ __forceinline__ void combine_item(const AttnArgs &a, const CombJob &j
     const int rows = min(kBM, job.N * G - job.mtile * kBM);
     const int rbase = row0 + grp * rpw;                 // this lane's first row in the tile
     const int npairs = max(0, min(rpw, rows - rbase)) * np;
-    const bool fast = job.W >= Gc;
-    const long long u_c = fast ? 0 : range_lo(c, job.W, Gc);
-    auto slot_of = [&](int p) -> long long {
-        if (p == 0) return job.first_slot;
-        return fast ? 2ll * (c + p) : 2ll * owner_of(u_c + p, job.W, Gc);
-    };
+    // piece p > 0: slot 0 of the p-th CTA with a non-empty range after CTA c
+    auto slot_of = [&](int p) -> long long { return p == 0 ? job.first_slot : 2ll * nonempty[p]; };
     float M = -INFINITY, L = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     int k = 0, p = 0;  // row and piece the fold is at
@@ -188,43 +202,44 @@ __global__ void __launch_bounds__(kCombThreads, 3)
 attn_combine(AttnArgs a, int Gc) {
     pdl_enter();
     __shared__ CombJob s_job[kAttnMaxGrid];
-    __shared__ int s_np[kAttnMaxGrid], s_rpw[kAttnMaxGrid];
+    __shared__ int s_np[kAttnMaxGrid], s_rpw[kAttnMaxGrid], s_rank[kAttnMaxGrid];
+    __shared__ int s_ne[kAttnMaxGrid];  // the CTAs with a non-empty range, in order
     __shared__ int s_pre[kAttnMaxGrid + 1];
     __shared__ int s_w[kCombThreads / 32];
-    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int t = threadIdx.x;
     const int G = a.Hq / a.Hkv;
     constexpr int rows_per_group = kCombThreads / (D / 4);  // rows of an item with rpw = 1
+    // CTA t's job and whether its range is empty
+    CombJob j;
+    j.b = -1;
+    int ne = 0;
+    if (t < Gc) {
+        j = a.jobs[t];
+        s_job[t] = j;
+        const int2 rg = a.ranges[t];
+        ne = rg.y > rg.x;
+    }
+    int n_ne;
+    const int rank = block_excl_scan(ne, s_w, &n_ne);
+    if (t < Gc) {
+        s_rank[t] = rank;
+        if (ne) s_ne[rank] = t;
+    }
+    __syncthreads();
     // items of the job of CTA t
     int items = 0;
-    if (t < Gc) {
-        const CombJob j = a.jobs[t];
-        s_job[t] = j;
-        if (j.b >= 0) {
-            const int np = comb_np(j, t, Gc);
-            const int rpw = np <= 2 ? 4 : (np <= 4 ? 2 : 1);
-            const int rows = min(kBM, j.N * G - j.mtile * kBM);
-            const int per = rows_per_group * rpw;
-            s_np[t] = np;
-            s_rpw[t] = rpw;
-            items = (rows + per - 1) / per;
-        }
+    if (t < Gc && j.b >= 0) {
+        const int np = s_rank[j.c1] - rank + 1;  // CTAs t and c1 both hold a piece
+        const int rpw = np <= 2 ? 4 : (np <= 4 ? 2 : 1);
+        const int rows = min(kBM, j.N * G - j.mtile * kBM);
+        const int per = rows_per_group * rpw;
+        s_np[t] = np;
+        s_rpw[t] = rpw;
+        items = (rows + per - 1) / per;
     }
-    // exclusive prefix of the item counts (CTA order)
-    int x = items;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, x, o);
-        if (lane >= o) x += y;
-    }
-    if (lane == 31) s_w[warp] = x;
-    __syncthreads();
-    int before = 0, total = 0;
-#pragma unroll
-    for (int w = 0; w < kCombThreads / 32; ++w) {
-        before += w < warp ? s_w[w] : 0;
-        total += s_w[w];
-    }
-    if (t < Gc) s_pre[t] = before + x - items;
+    int total;
+    const int pre = block_excl_scan(items, s_w, &total);
+    if (t < Gc) s_pre[t] = pre;
     if (t == 0) s_pre[Gc] = total;
     __syncthreads();
     for (int it = blockIdx.x; it < total; it += gridDim.x) {
@@ -236,7 +251,7 @@ attn_combine(AttnArgs a, int Gc) {
         }
         const int c = lo;
         const int row0 = (it - s_pre[c]) * rows_per_group * s_rpw[c];
-        combine_item<D>(a, s_job[c], c, s_np[c], Gc, row0, s_rpw[c]);
+        combine_item<D>(a, s_job[c], s_np[c], s_ne + s_rank[c], row0, s_rpw[c]);
     }
 }
 
@@ -288,6 +303,7 @@ extern "C" size_t rs_tree_verify_attn_workspace_size(int B, int R, int Hq, int H
     cv.take<float>(2 * Gc * kBM);
     cv.take<float>(2 * Gc * kBM);
     cv.take<CombJob>(Gc);
+    cv.take<int2>(Gc);
     return cv.used();
 }
 
@@ -334,6 +350,7 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     a.part_m = cv.take<float>(2 * (size_t)Gc * kBM);
     a.part_l = cv.take<float>(2 * (size_t)Gc * kBM);
     a.jobs = cv.take<CombJob>((size_t)Gc);
+    a.ranges = cv.take<int2>((size_t)Gc);
     a.B = B;
     a.Hq = Hq;
     a.Hkv = Hkv;

@@ -51,14 +51,25 @@ constexpr int kSmemBar = kSmemV + kNS * kTileBytes;
 constexpr int kNumBars = 4 * kNS + 12;
 constexpr int kSmemMisc = kSmemBar + kNumBars * 8;  // tmem base, abort flag
 constexpr int kSmemPref = kSmemMisc + 16;
-constexpr int kAttnMaxB = 4096;
+constexpr int kAttnMaxB = 3840;  // requests per call (the two prefixes over them live in shared memory)
 constexpr int kAttnMaxGrid = 256;  // CTAs (one per SM, at most this many)
 constexpr long long kWaitLimit = 4000000000ll;     // clock cycles (~2 s)
 constexpr uint32_t kTmemCols = 512;
 // TMEM columns: O [0, 128), S/P buffers [128, 256) and [256, 384), Q [384, 448)
 constexpr uint32_t kTmO = 0, kTmS = 128, kTmQ = 384;
 
-inline size_t attn_smem_bytes(int B) { return 1024 + kSmemPref + (size_t)(B + 1) * sizeof(int); }
+// In the split of the work over the CTAs each segment (request, KV head, row
+// tile) costs its KV tiles plus beta = min(kSegCostMax, W / (2 G)) tiles (W
+// units, G CTAs): a piece boundary (Q loaded, pipeline restarted, epilogue)
+// costs several tiles' worth, so CTAs whose ranges cut many short segments
+// were the stragglers.  The cap keeps small launches (a few units per CTA)
+// close to an even split of the units, and launches with long ranges
+// (>= kSegCostOff units per CTA, where a boundary is a small part of a range
+// and every CTA has about the same number of pieces) keep the even split.
+constexpr int kSegCostMax = 8;
+constexpr int kSegCostOff = 128;
+// unit and segment prefixes over the requests: 2 (B + 1) ints after kSmemPref
+inline size_t attn_smem_bytes(int B) { return 1024 + kSmemPref + 2 * (size_t)(B + 1) * sizeof(int); }
 
 struct ReqInfo {
     int units;  // Hkv * mt * nt, 0 for a rejected request
@@ -86,6 +97,7 @@ struct AttnArgs {
     const uint32_t *anc;
     float *part_o, *part_m, *part_l;
     CombJob *jobs;  // [gridDim.x]
+    int2 *ranges;   // [gridDim.x]: each CTA's unit range [x, y)
     int kv_stream;  // the launch's K/V is large next to L2: stream tiles read once
     int B, Hq, Hkv, D;
     float scale;
@@ -94,41 +106,60 @@ struct AttnArgs {
 };
 
 // ------------------------------------------------------------------ schedule
-// Exclusive prefix of per-request units into s_pref[0..B] (s_pref[B] = W).
-__device__ inline void unit_prefix(const ReqInfo *__restrict__ info, int B, int *s_pref) {
-    __shared__ int s_carry;
-    __shared__ int s_w[32];
-    if (threadIdx.x == 0) s_carry = 0;
+// Exclusive prefixes over the requests of their units (s_pref[0..B],
+// s_pref[B] = W) and of their segments (s_spref).
+__device__ inline void unit_prefix(const ReqInfo *__restrict__ info, int B, int *s_pref, int *s_spref) {
+    __shared__ int s_carry[2];
+    __shared__ int s_w[2][32];
+    if (threadIdx.x == 0) s_carry[0] = s_carry[1] = 0;
     __syncthreads();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nw = (blockDim.x + 31) >> 5;
     for (int base = 0; base < B; base += blockDim.x) {
-        int i = base + threadIdx.x;
-        int v = i < B ? info[i].units : 0;
-        int x = v;
-        for (int o = 1; o < 32; o <<= 1) {
-            int y = __shfl_up_sync(0xffffffffu, x, o);
-            if (lane >= o) x += y;
+        const int i = base + threadIdx.x;
+        int v[2] = {0, 0};
+        if (i < B) {
+            const ReqInfo ri = info[i];
+            v[0] = ri.units;
+            v[1] = ri.nt > 0 ? ri.units / ri.nt : 0;
         }
-        if (lane == 31) s_w[warp] = x;
+        int x[2] = {v[0], v[1]};
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xffffffffu, x[k], o);
+                if (lane >= o) x[k] += y;
+            }
+            if (lane == 31) s_w[k][warp] = x[k];
+        }
         __syncthreads();
         if (warp == 0) {
-            int w = lane < nw ? s_w[lane] : 0;
-            int z = w;
-            for (int o = 1; o < 32; o <<= 1) {
-                int y = __shfl_up_sync(0xffffffffu, z, o);
-                if (lane >= o) z += y;
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const int w = lane < nw ? s_w[k][lane] : 0;
+                int z = w;
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int y = __shfl_up_sync(0xffffffffu, z, o);
+                    if (lane >= o) z += y;
+                }
+                s_w[k][lane] = z - w;
             }
-            s_w[lane] = z - w;
         }
         __syncthreads();
-        int incl = s_carry + s_w[warp] + x;
-        if (i < B) s_pref[i + 1] = incl;
+        const int incl0 = s_carry[0] + s_w[0][warp] + x[0];
+        const int incl1 = s_carry[1] + s_w[1][warp] + x[1];
+        if (i < B) {
+            s_pref[i + 1] = incl0;
+            s_spref[i + 1] = incl1;
+        }
         __syncthreads();
-        if (threadIdx.x == blockDim.x - 1) s_carry = incl;
+        if (threadIdx.x == blockDim.x - 1) {
+            s_carry[0] = incl0;
+            s_carry[1] = incl1;
+        }
         __syncthreads();
     }
-    if (threadIdx.x == 0) s_pref[0] = 0;
+    if (threadIdx.x == 0) s_pref[0] = s_spref[0] = 0;
     __syncthreads();
 }
 
@@ -143,9 +174,48 @@ __device__ __forceinline__ int find_req(const int *s_pref, int B, long long u) {
     return lo;
 }
 
-__device__ __forceinline__ long long range_lo(long long c, long long W, long long G) { return c * W / G; }
-__device__ __forceinline__ long long owner_of(long long u, long long W, long long G) {
-    return ((u + 1) * G - 1) / W;
+// The work split.  Cost positions: request b's segments occupy
+// [cost(b), cost(b + 1)), cost(b) = s_pref[b] + beta s_spref[b], nt + beta
+// each; CTA c takes [c C / G, (c + 1) C / G) (C = cost(B)).  A position in a
+// segment's first beta maps to the segment's first unit, so the ranges are
+// unit ranges that tile [0, W) in order (some may be empty).
+struct Split {
+    const int *pref, *spref;
+    int B, beta, G;
+    __device__ __forceinline__ int cost(int b) const { return pref[b] + beta * spref[b]; }
+    __device__ __forceinline__ long long unit_at(int x) const {
+        if (x >= cost(B)) return pref[B];
+        int lo = 0, hi = B - 1;  // last b with cost(b) <= x: a request with units
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (cost(mid) <= x) lo = mid;
+            else hi = mid - 1;
+        }
+        const int nt = (pref[lo + 1] - pref[lo]) / (spref[lo + 1] - spref[lo]);
+        const int local = x - cost(lo);
+        const int seg = local / (nt + beta);
+        const int off = local - seg * (nt + beta) - beta;
+        return pref[lo] + seg * nt + (off > 0 ? off : 0);
+    }
+    __device__ __forceinline__ long long range_lo(long long c) const {
+        return unit_at((int)(c * cost(B) / G));
+    }
+    // The CTA holding the last unit of segment [s0, s1) of request b: that
+    // unit's cost position x lies in CTA c's cost interval for
+    // c = ((x + 1) G - 1) / C, and the unit ranges follow the cost intervals.
+    __device__ __forceinline__ long long owner_of_seg_end(int b, long long s0, long long s1) const {
+        const int nt = (int)(s1 - s0);
+        const int seg = (int)((s0 - pref[b]) / nt);
+        const long long x = (long long)cost(b) + (long long)(seg + 1) * (nt + beta) - 1;
+        return ((x + 1) * G - 1) / cost(B);
+    }
+};
+__device__ __forceinline__ Split make_split(const int *s_pref, const int *s_spref, int B, int G) {
+    const int W = s_pref[B];
+    int beta = W / (2 * G);
+    if (beta > kSegCostMax) beta = kSegCostMax;
+    if (W >= kSegCostOff * G) beta = 0;
+    return Split{s_pref, s_spref, B, beta, G};
 }
 
 struct Piece {
@@ -234,6 +304,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + kSmemMisc);
     volatile int *s_abort = reinterpret_cast<volatile int *>(smem + kSmemMisc + 4);
     int *s_pref = reinterpret_cast<int *>(smem + kSmemPref);
+    int *s_spref = s_pref + (a.B + 1);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     if (tid == 0) {
@@ -262,12 +333,13 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
         prefetch_tmap(&tmv);
     }
     pdl_wait_prev();  // the prologue above touches no global memory
-    unit_prefix(info, a.B, s_pref);  // contains __syncthreads
+    unit_prefix(info, a.B, s_pref, s_spref);  // contains __syncthreads
     tc_fence_after();
     const uint32_t tmem = *s_tmem;
     const long long W = s_pref[a.B];
     const long long Gc = gridDim.x, c = blockIdx.x;
-    const long long u0 = range_lo(c, W, Gc), u1 = range_lo(c + 1, W, Gc);
+    const Split split = make_split(s_pref, s_spref, a.B, (int)Gc);
+    const long long u0 = split.range_lo(c), u1 = split.range_lo(c + 1);
     const int G = a.Hq / a.Hkv;
     constexpr uint32_t kTileTx = (uint32_t)kBN * D * 2;
     constexpr int kKB = D / 64;  // 64-column swizzle blocks per row
@@ -332,10 +404,11 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                     job.n0 = a.node_off[pl.b];
                     job.N = a.node_off[pl.b + 1] - job.n0;
                     job.first_slot = (int)(2 * c + (pl.seg_start > u0 ? 1 : 0));
-                    job.c1 = (int)owner_of(pl.seg_end - 1, W, Gc);
+                    job.c1 = (int)split.owner_of_seg_end(pl.b, pl.seg_start, pl.seg_end);
                 }
             }
             a.jobs[c] = job;
+            a.ranges[c] = make_int2((int)u0, (int)u1);
         }
     } else if (warp == kMmaWarp) {
         // ---------------------------------------------------------- MMA issuer
