@@ -330,6 +330,8 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     RS_CHECK_ARG(kv_rows == 0 || (k && v), "rs_tree_verify_attn: null KV pointer");
     RS_CHECK_ARG((((uintptr_t)k | (uintptr_t)v | (uintptr_t)q) & 15) == 0,
                  "rs_tree_verify_attn: q, k and v must be 16-byte aligned");
+    RS_CHECK_ARG((((uintptr_t)out | (uintptr_t)workspace) & 15) == 0,
+                 "rs_tree_verify_attn: out and workspace must be 16-byte aligned");
     if (B == 0) return RS_OK;
     const size_t need = rs_tree_verify_attn_workspace_size(B, R, Hq, Hkv, D);
     if (workspace_bytes < need || !workspace) {
@@ -360,6 +362,7 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     a.lse = lse;
     a.status = status;
     a.kv_stream = 2.0 * (double)kv_rows * Hkv * D * 2 > 0.5 * (double)l2_bytes();
+    a.out32 = (((uintptr_t)out | (uintptr_t)a.part_o) & 31) == 0;
     cudaStream_t st = (cudaStream_t)stream;
 
     // a map over an empty KV cache is never dereferenced: point it at q
