@@ -395,9 +395,9 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     }
     const size_t smem = attn_smem_bytes(B);
     if (D == 128)
-        launch_full(attn_tc_kernel<128>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
+        launch_pdl(attn_tc_kernel<128>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
     else
-        launch_full(attn_tc_kernel<64>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
+        launch_pdl(attn_tc_kernel<64>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/main");
     // a full launch: combine blocks parked early beside the attention CTAs
     // (programmatic launch) measured slower on the batched workload
