@@ -68,6 +68,29 @@ def test_attention_rejects_bad_trees_and_keeps_the_rest():
         assert np.abs(got - ref["out"]).max() < 1e-2
 
 
+@pytest.mark.parametrize("B,ctx_hi,D", [(3840, 12, 64), (300, 400, 128)])
+def test_attention_many_requests(B, ctx_hi, D):
+    # the largest request count a call takes (two prefixes over the requests
+    # in shared memory), and a few hundred short requests whose segments the
+    # cost-weighted split spreads over the CTAs (some ranges empty)
+    rng = np.random.default_rng(B)
+    Hq, Hkv = 2, 1
+    trees = []
+    for _ in range(B):
+        n = int(rng.integers(1, 6))
+        trees.append([-1] + [int(rng.integers(0, i)) for i in range(1, n)])
+    S = [int(x) for x in rng.integers(0, ctx_hi, B)]
+    inp = _attn_inputs(rng, Hq, Hkv, D, S, trees)
+    out, lse, status = _run_attn(*inp, Hq, Hkv, D, D ** -0.5)
+    assert (status == 0).all()
+    q, k, v, kv_off, ctx, node_off, parents = inp
+    R = int(node_off[-1])
+    rows = [(n, h) for n in range(0, R, max(1, R // 600)) for h in range(Hq)]
+    ref = oracle.tree_attn(q, k, v, kv_off, ctx, node_off, parents, Hq, Hkv, D, D ** -0.5, rows=rows)
+    got = np.stack([out[n, h] for n, h in rows])
+    assert np.abs(got - ref["out"].reshape(len(rows), D)).max() < 1e-2
+
+
 def test_attention_single_node_and_tile_straddling_tree():
     rng = np.random.default_rng(1)
     Hq, Hkv, D = 6, 3, 64
