@@ -312,7 +312,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
         for (int s = 0; s < kNS; ++s) {
             mbar_init(&kfull[s], 1);
             mbar_init(&vfull[s], 1);
-            mbar_init(&kempty[s], 1);
+            mbar_init(&kempty[s], kSoftThreads);  // released by the softmax warps
             mbar_init(&vempty[s], 1);
         }
         for (int s = 0; s < 2; ++s) {
@@ -432,7 +432,6 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                     umma_ts(d_s, q_tm + kk * 8, sdesc_sw128(k_addr + off, 16, 1024), idS, kk > 0);
                 }
                 umma_commit(&sfull[gt & 1]);
-                umma_commit(&kempty[st]);
                 return true;
             };
             for (long long u = u0; u < u1 && ok; ++piece) {
@@ -530,6 +529,9 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                 const int jt = pc.j0 + tl;
                 if (!(ok = warp_wait(&sfull[buf], (uint32_t)((gt >> 1) & 1), s_abort))) break;
                 tc_fence_after();
+                // S of this tile is complete, so its K stage is free: released
+                // here rather than by a second commit on the MMA thread
+                warp_arrive(&kempty[(int)(gt % kNS)]);
                 const uint32_t s_tm = tmem + lane_off + kTmS + (uint32_t)buf * 128;
                 float s[64];
                 {  // both halves in flight, one wait
