@@ -123,6 +123,12 @@ __device__ __forceinline__ float4 ldg_stream4(const float4 *p) {
                  : "l"(p));
     return r;
 }
+// 256-bit variant (p 32-byte aligned).
+__device__ __forceinline__ void ldg_stream8(const float *p, float (&r)[8]) {
+    asm volatile("ld.global.nc.L1::no_allocate.v8.f32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=f"(r[0]), "=f"(r[1]), "=f"(r[2]), "=f"(r[3]), "=f"(r[4]), "=f"(r[5]), "=f"(r[6]), "=f"(r[7])
+                 : "l"(p));
+}
 __device__ __forceinline__ float ldg_stream(const float *p) {
     float r;
     asm volatile("ld.global.nc.L1::no_allocate.f32 %0, [%1];" : "=f"(r) : "l"(p));

@@ -55,7 +55,9 @@ __device__ __forceinline__ float ex2f_approx(float x) {
     return y;
 }
 
-template <bool kVec>
+// kW: logits per load (8: V % 8 == 0 and 32-byte aligned logits; 4: V % 4 ==
+// 0 and 16-byte alignment; else 1).
+template <int kW>
 __global__ void __launch_bounds__(kGateThreads)
 entropy_partial(const float *__restrict__ logits, int V, int nchunks, Ent3 *__restrict__ part) {
     pdl_enter();
@@ -67,7 +69,19 @@ entropy_partial(const float *__restrict__ logits, int V, int nchunks, Ent3 *__re
     const int tid = threadIdx.x;
 
     float v[kGateVpt];
-    if (kVec) {
+    if (kW == 8) {
+        // 4 x 256-bit loads per thread, each iteration a contiguous 8 KB sweep
+#pragma unroll
+        for (int j = 0; j < kGateVpt / 8; ++j) {
+            const int idx = c0 + (j * kGateThreads + tid) * 8;
+            float x[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) x[k] = -INFINITY;
+            if (idx < V) ldg_stream8(row + idx, x);  // V % 8 == 0: whole groups of 8
+#pragma unroll
+            for (int k = 0; k < 8; ++k) v[8 * j + k] = x[k];
+        }
+    } else if (kW == 4) {
         // 8 x float4 per thread, each iteration a contiguous 4 KB sweep
 #pragma unroll
         for (int j = 0; j < kGateVpt / 4; ++j) {
@@ -260,13 +274,17 @@ rs_status launch_gate(const char *who, const float *logits, int R, int V, int nc
             set_error("%s: R*chunks too large", who);
             return RS_ERR_INVALID_ARG;
         }
-        const bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
-        if (vec)
-            launch_pdl(entropy_partial<true>, dim3((unsigned)blocks), dim3(kGateThreads), 0, st, logits, V,
-                nchunks, part);
+        const int w = (V % 8 == 0 && ((uintptr_t)logits & 31) == 0) ? 8
+                      : (V % 4 == 0 && ((uintptr_t)logits & 15) == 0) ? 4 : 1;
+        if (w == 8)
+            launch_pdl(entropy_partial<8>, dim3((unsigned)blocks), dim3(kGateThreads), 0, st, logits, V, nchunks,
+                part);
+        else if (w == 4)
+            launch_pdl(entropy_partial<4>, dim3((unsigned)blocks), dim3(kGateThreads), 0, st, logits, V, nchunks,
+                part);
         else
-            launch_pdl(entropy_partial<false>, dim3((unsigned)blocks), dim3(kGateThreads), 0, st, logits, V,
-                nchunks, part);
+            launch_pdl(entropy_partial<1>, dim3((unsigned)blocks), dim3(kGateThreads), 0, st, logits, V, nchunks,
+                part);
         RS_CHECK_LAUNCH(who);
         launch_pdl(entropy_merge, dim3((R + kMergeThreads / 32 - 1) / (kMergeThreads / 32)), dim3(kMergeThreads),
             0, st, part, nchunks, R, entropy);
