@@ -46,10 +46,10 @@ __device__ __forceinline__ float ex2f(float x) {
 }
 
 // This thread's 32 logits of chunk c0 (ids >= V read as -inf).
-template <bool kVec>
+template <int kW>
 __device__ __forceinline__ void load32(const float *__restrict__ row, int V, int c0, float (&z)[kSmpVpt]) {
     const int base = c0 + threadIdx.x * kSmpVpt;
-    if (kVec && base + kSmpVpt <= V) {
+    if (kW >= 4 && base + kSmpVpt <= V) {
         const float4 *p = reinterpret_cast<const float4 *>(row + base);
 #pragma unroll
         for (int q = 0; q < kSmpVpt / 4; ++q) {
@@ -73,16 +73,30 @@ __device__ __forceinline__ void load32(const float *__restrict__ row, int V, int
 // way, so the per-thread sums do not depend on the path.
 constexpr int kSmpPadded = kSmpChunk + kSmpChunk / 8;  // 36 floats per thread
 
-template <bool kVec>
+// kW: logits per streaming load (8: V % 8 == 0 and 32-byte aligned logits;
+// 4: V % 4 == 0 and 16-byte alignment; 1: no staging).
+template <int kW>
 __device__ __forceinline__ void load32_staged(const float *__restrict__ row, int V, int c0, float *s_buf,
                                               float (&z)[kSmpVpt]) {
-    if (kVec && c0 + kSmpChunk <= V) {  // uniform over the CTA
+    if (kW >= 4 && c0 + kSmpChunk <= V) {  // uniform over the CTA
         const int tid = threadIdx.x;
+        if (kW == 8) {
 #pragma unroll
-        for (int j = 0; j < kSmpVpt / 4; ++j) {
-            const int e = 4 * (j * kSmpThreads + tid);
-            const float4 x = ldg_stream4(reinterpret_cast<const float4 *>(row + c0 + e));
-            *reinterpret_cast<float4 *>(s_buf + e + 4 * (e >> 5)) = x;
+            for (int j = 0; j < kSmpVpt / 8; ++j) {
+                const int e = 8 * (j * kSmpThreads + tid);  // 8 ids in one padded 32-group
+                float x[8];
+                ldg_stream8(row + c0 + e, x);
+                float4 *d = reinterpret_cast<float4 *>(s_buf + e + 4 * (e >> 5));
+                d[0] = make_float4(x[0], x[1], x[2], x[3]);
+                d[1] = make_float4(x[4], x[5], x[6], x[7]);
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < kSmpVpt / 4; ++j) {
+                const int e = 4 * (j * kSmpThreads + tid);
+                const float4 x = ldg_stream4(reinterpret_cast<const float4 *>(row + c0 + e));
+                *reinterpret_cast<float4 *>(s_buf + e + 4 * (e >> 5)) = x;
+            }
         }
         __syncthreads();
         const float4 *p = reinterpret_cast<const float4 *>(s_buf + tid * (kSmpVpt + 4));
@@ -95,7 +109,7 @@ __device__ __forceinline__ void load32_staged(const float *__restrict__ row, int
             z[4 * q + 3] = x.w;
         }
     } else {
-        load32<kVec>(row, V, c0, z);
+        load32<kW>(row, V, c0, z);
     }
 }
 
@@ -134,7 +148,7 @@ __device__ __forceinline__ float block_incl_scan(float v, float *s_w, float *tot
     return before + x;
 }
 
-template <bool kVec>
+template <int kW>
 __global__ void __launch_bounds__(kSmpThreads)
 sample_partial(const float *__restrict__ logits, int V, int nchunks, float scale, ChunkMass *__restrict__ part) {
     pdl_enter();
@@ -143,7 +157,7 @@ sample_partial(const float *__restrict__ logits, int V, int nchunks, float scale
     const int r = blockIdx.x / nchunks, c = blockIdx.x - r * nchunks;
     const float *row = logits + (long long)r * V;
     float z[kSmpVpt];
-    load32_staged<kVec>(row, V, c * kSmpChunk, s_buf, z);
+    load32_staged<kW>(row, V, c * kSmpChunk, s_buf, z);
     float mx = -INFINITY;
 #pragma unroll
     for (int j = 0; j < kSmpVpt; ++j) mx = fmaxf(mx, z[j]);
@@ -159,7 +173,7 @@ sample_partial(const float *__restrict__ logits, int V, int nchunks, float scale
     if (threadIdx.x == 0) part[blockIdx.x] = ChunkMass{m, tot};
 }
 
-template <bool kVec>
+template <int kW>
 __global__ void __launch_bounds__(kSmpThreads)
 sample_pick(const float *__restrict__ logits, int V, int nchunks, float scale, const ChunkMass *__restrict__ part,
             const float *__restrict__ uniforms, int32_t *__restrict__ draw) {
@@ -236,7 +250,7 @@ sample_pick(const float *__restrict__ logits, int V, int nchunks, float scale, c
     const float nb = -m * scale;
     const float *row = logits + (long long)r * V;
     float z[kSmpVpt];
-    load32_staged<kVec>(row, V, c * kSmpChunk, s_buf, z);
+    load32_staged<kW>(row, V, c * kSmpChunk, s_buf, z);
     float s = 0.f;
 #pragma unroll
     for (int j = 0; j < kSmpVpt; ++j) s += ex2f(fmaf(z[j], scale, nb));
@@ -383,19 +397,17 @@ extern "C" rs_status rs_tree_sample(const float *logits, int R, int V, const int
     ChunkMass *part = static_cast<ChunkMass *>(workspace);
     const float scale = kL2E / temperature;
     if (R > 0) {
-        const bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
+        const int w = (V % 8 == 0 && ((uintptr_t)logits & 31) == 0) ? 8
+                      : (V % 4 == 0 && ((uintptr_t)logits & 15) == 0) ? 4 : 1;
         const unsigned blocks = (unsigned)((long long)R * nchunks);
-        if (vec)
-            launch_pdl(sample_partial<true>, dim3(blocks), dim3(kSmpThreads), 0, st, logits, V, nchunks, scale, part);
-        else
-            launch_pdl(sample_partial<false>, dim3(blocks), dim3(kSmpThreads), 0, st, logits, V, nchunks, scale, part);
+        const dim3 blk(kSmpThreads);
+        if (w == 8) launch_pdl(sample_partial<8>, dim3(blocks), blk, 0, st, logits, V, nchunks, scale, part);
+        else if (w == 4) launch_pdl(sample_partial<4>, dim3(blocks), blk, 0, st, logits, V, nchunks, scale, part);
+        else launch_pdl(sample_partial<1>, dim3(blocks), blk, 0, st, logits, V, nchunks, scale, part);
         RS_CHECK_LAUNCH("rs_tree_sample/partial");
-        if (vec)
-            launch_pdl(sample_pick<true>, dim3(R), dim3(kSmpThreads), 0, st, logits, V, nchunks, scale, part, uniforms,
-                draw);
-        else
-            launch_pdl(sample_pick<false>, dim3(R), dim3(kSmpThreads), 0, st, logits, V, nchunks, scale, part, uniforms,
-                draw);
+        if (w == 8) launch_pdl(sample_pick<8>, dim3(R), blk, 0, st, logits, V, nchunks, scale, part, uniforms, draw);
+        else if (w == 4) launch_pdl(sample_pick<4>, dim3(R), blk, 0, st, logits, V, nchunks, scale, part, uniforms, draw);
+        else launch_pdl(sample_pick<1>, dim3(R), blk, 0, st, logits, V, nchunks, scale, part, uniforms, draw);
         RS_CHECK_LAUNCH("rs_tree_sample/pick");
     }
     if (B > 0) {
