@@ -115,9 +115,7 @@ struct RowsShared {
 //     candidates before it in the total order).  If ties at T overflow the
 //     buffer, every warp ranks its own logits by beta "best after the
 //     previous winner" rounds and warp 0 merges the eight lists (exact too).
-// kW: logits per load (8 for 256-bit loads when V % 8 == 0 and the logits
-// are 32-byte aligned, 4 for V % 4 == 0 and 16-byte alignment, else 1).
-template <int kW, bool kEnt>
+template <bool kVec, bool kEnt>
 __global__ void __launch_bounds__(kAccThreads, 4)
 accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *__restrict__ cand,
             MS *__restrict__ part) {
@@ -133,24 +131,11 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
 
     // logit id of register j (ids >= V are padding, held as -inf)
     auto id_of = [&](int j) -> int {
-        if (kW == 8) return c0 + ((j >> 3) * kAccThreads + tid) * 8 + (j & 7);
-        if (kW == 4) return c0 + ((j >> 2) * kAccThreads + tid) * 4 + (j & 3);
+        if (kVec) return c0 + ((j >> 2) * kAccThreads + tid) * 4 + (j & 3);
         return c0 + j * kAccThreads + tid;
     };
     float v[kAccVpt];
-    if (kW == 8) {
-        const bool inside = c0 + kAccChunk <= V;
-#pragma unroll
-        for (int j = 0; j < kAccVpt / 8; ++j) {
-            const int off = c0 + (j * kAccThreads + tid) * 8;
-            float x[8];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) x[k] = -INFINITY;
-            if (inside || off < V) ldg_stream8(row + off, x);  // V % 8 == 0: whole groups of 8
-#pragma unroll
-            for (int k = 0; k < 8; ++k) v[8 * j + k] = x[k];
-        }
-    } else if (kW == 4) {
+    if (kVec) {
         const bool inside = c0 + kAccChunk <= V;
 #pragma unroll
         for (int j = 0; j < kAccVpt / 4; ++j) {
@@ -669,17 +654,18 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
     if (R > 0) {
         const long long blocks = (long long)R * nchunks;
         RS_CHECK_ARG(blocks < (1ll << 30), "rs_accept: R*chunks too large");
-        const int w = (V % 8 == 0 && ((uintptr_t)logits & 31) == 0) ? 8
-                      : (V % 4 == 0 && ((uintptr_t)logits & 15) == 0) ? 4 : 1;
+        const bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
         const bool ent = entropy != nullptr;
         const dim3 grid((unsigned)blocks);
-        const dim3 blk(kAccThreads);
-        if (w == 8 && ent) launch_pdl(accept_rows<8, true>, grid, blk, 0, st, logits, V, nchunks, p.beta, cand, part);
-        else if (w == 8) launch_pdl(accept_rows<8, false>, grid, blk, 0, st, logits, V, nchunks, p.beta, cand, part);
-        else if (w == 4 && ent) launch_pdl(accept_rows<4, true>, grid, blk, 0, st, logits, V, nchunks, p.beta, cand, part);
-        else if (w == 4) launch_pdl(accept_rows<4, false>, grid, blk, 0, st, logits, V, nchunks, p.beta, cand, part);
-        else if (ent) launch_pdl(accept_rows<1, true>, grid, blk, 0, st, logits, V, nchunks, p.beta, cand, part);
-        else launch_pdl(accept_rows<1, false>, grid, blk, 0, st, logits, V, nchunks, p.beta, cand, part);
+        if (vec && ent)
+            launch_pdl(accept_rows<true, true>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand, part);
+        else if (vec)
+            launch_pdl(accept_rows<true, false>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand, part);
+        else if (ent)
+            launch_pdl(accept_rows<false, true>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand, part);
+        else
+            launch_pdl(accept_rows<false, false>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand,
+                part);
         RS_CHECK_LAUNCH("rs_accept/accept_rows");
         launch_pdl(accept_merge, dim3((R + kMergeThreads / 32 - 1) / (kMergeThreads / 32)), dim3(kMergeThreads),
             0, st, cand, part, nchunks, p.beta, R, argmax, topk, lse, entropy, rowmax);
