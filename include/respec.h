@@ -219,8 +219,7 @@ rs_status rs_match_scan(const int32_t *tokens, const int64_t *tok_off, int B,
  *   head h / (Hq / Hkv)); scale > 0 is the softmax scale (1/sqrt(D) usually).
  *   out      [R, Hq, D] fp32 attention outputs;  lse [R, Hq] fp32 natural-log
  *            sum of exp(scale * q.k) over the attended keys.  out and the
- *            workspace must be 16-byte aligned (32-byte alignment of both
- *            lets the kernel use 256-bit stores).
+ *            workspace must be 16-byte aligned.
  *   status   [B]: RS_ST_BAD_TREE / RS_ST_TOO_LARGE for a malformed request
  *            (its out/lse rows are zeroed).
  * QK^T and PV run on the tensor cores with fp32 accumulation.

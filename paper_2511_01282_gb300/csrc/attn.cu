@@ -219,11 +219,20 @@ attn_combine(AttnArgs a, int Gc) {
         const int2 rg = a.ranges[t];
         ne = rg.y > rg.x;
     }
-    int n_ne;
-    const int rank = block_excl_scan(ne, s_w, &n_ne);
-    if (t < Gc) {
-        s_rank[t] = rank;
-        if (ne) s_ne[rank] = t;
+    int rank;
+    if (!__syncthreads_or(t < Gc && !ne)) {  // every range non-empty (the usual case): no scan
+        rank = t;
+        if (t < Gc) {
+            s_rank[t] = t;
+            s_ne[t] = t;
+        }
+    } else {
+        int n_ne;
+        rank = block_excl_scan(ne, s_w, &n_ne);
+        if (t < Gc) {
+            s_rank[t] = rank;
+            if (ne) s_ne[rank] = t;
+        }
     }
     __syncthreads();
     // items of the job of CTA t
@@ -362,7 +371,6 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     a.lse = lse;
     a.status = status;
     a.kv_stream = 2.0 * (double)kv_rows * Hkv * D * 2 > 0.5 * (double)l2_bytes();
-    a.out32 = (((uintptr_t)out | (uintptr_t)a.part_o) & 31) == 0;
     cudaStream_t st = (cudaStream_t)stream;
 
     // a map over an empty KV cache is never dereferenced: point it at q
@@ -395,9 +403,9 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     }
     const size_t smem = attn_smem_bytes(B);
     if (D == 128)
-        launch_pdl(attn_tc_kernel<128>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
+        launch_full(attn_tc_kernel<128>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
     else
-        launch_pdl(attn_tc_kernel<64>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
+        launch_full(attn_tc_kernel<64>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/main");
     // a full launch: combine blocks parked early beside the attention CTAs
     // (programmatic launch) measured slower on the batched workload

@@ -99,7 +99,6 @@ struct AttnArgs {
     CombJob *jobs;  // [gridDim.x]
     int2 *ranges;   // [gridDim.x]: each CTA's unit range [x, y)
     int kv_stream;  // the launch's K/V is large next to L2: stream tiles read once
-    int out32;      // out and the partial slots are 32-byte aligned: 256-bit stores
     int B, Hq, Hkv, D;
     float scale;
     float *out, *lse;
@@ -199,6 +198,7 @@ struct Split {
         return pref[lo] + seg * nt + (off > 0 ? off : 0);
     }
     __device__ __forceinline__ long long range_lo(long long c) const {
+        if (beta == 0) return c * pref[B] / G;  // an even split of the units
         return unit_at((int)(c * cost(B) / G));
     }
     // The CTA holding the last unit of segment [s0, s1) of request b: that
@@ -636,23 +636,13 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
             for (int ch = 0; ch < kHalfO / 32; ++ch) {
                 const int col = hw * kHalfO + ch * 32;
                 if (valid) {
-                    float *dst = pc.final ? a.out + orow * D + col : a.part_o + prow * D + col;
-                    if (a.out32) {  // whole 32-byte sectors per lane: half the store instructions
+                    float4 *dst = pc.final ? reinterpret_cast<float4 *>(a.out + orow * D + col)
+                                           : reinterpret_cast<float4 *>(a.part_o + prow * D + col);
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            float v[8];
-#pragma unroll
-                            for (int k = 0; k < 8; ++k) v[k] = __uint_as_float(xo[ch][8 * e + k]) * f;
-                            st_global_v8(dst + 8 * e, v);
-                        }
-                    } else {
-                        float4 *d4 = reinterpret_cast<float4 *>(dst);
-#pragma unroll
-                        for (int e = 0; e < 8; ++e)
-                            d4[e] = make_float4(__uint_as_float(xo[ch][4 * e]) * f, __uint_as_float(xo[ch][4 * e + 1]) * f,
-                                                __uint_as_float(xo[ch][4 * e + 2]) * f,
-                                                __uint_as_float(xo[ch][4 * e + 3]) * f);
-                    }
+                    for (int e = 0; e < 8; ++e)
+                        dst[e] = make_float4(__uint_as_float(xo[ch][4 * e]) * f, __uint_as_float(xo[ch][4 * e + 1]) * f,
+                                             __uint_as_float(xo[ch][4 * e + 2]) * f,
+                                             __uint_as_float(xo[ch][4 * e + 3]) * f);
                 }
             }
             if (valid && hw == 0) {

@@ -120,13 +120,6 @@ __device__ __forceinline__ void tc_fence_after() {
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
-// One 256-bit global store (p 32-byte aligned).
-__device__ __forceinline__ void st_global_v8(float *p, const float (&v)[8]) {
-    asm volatile("st.global.v8.f32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "f"(v[0]), "f"(v[1]), "f"(v[2]),
-                 "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7])
-                 : "memory");
-}
-
 // After tcgen05.wait::ld: an empty asm that "redefines" the loaded registers,
 // so that no use of them can be scheduled above the wait.
 __device__ __forceinline__ void tmem_regs_ready(uint32_t (&r)[32]) {
