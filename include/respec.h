@@ -65,7 +65,9 @@ typedef enum {
 #define RS_ST_BAD_POS    4  /* a selected position lies outside the buffer     */
 #define RS_ST_TOO_LARGE  8  /* more than RS_MAX_NODES tree nodes               */
 #define RS_ST_TIMEOUT   16  /* a pipeline wait inside a kernel gave up (bounded
-                               wait, ~2 s); the request's outputs are invalid   */
+                               wait, ~2 s; the environment variable
+                               RS_DEBUG_WAIT_LIMIT, in clock cycles, shortens it
+                               for tests); the request's outputs are invalid   */
 
 /* -------------------------------------------------------------- parameters */
 /* Hyper-parameters of Algorithm 1 (Require line), Eq. 6-7 and Section 3.4.

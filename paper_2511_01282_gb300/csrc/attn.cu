@@ -21,6 +21,7 @@
 #include <math.h>
 
 #include <algorithm>
+#include <cstdlib>
 
 #include <mutex>
 
@@ -371,6 +372,13 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     a.lse = lse;
     a.status = status;
     a.kv_stream = 2.0 * (double)kv_rows * Hkv * D * 2 > 0.5 * (double)l2_bytes();
+    // a test hook: RS_DEBUG_WAIT_LIMIT (clock cycles) shortens every pipeline
+    // wait so that the time-out path can be exercised
+    a.wait_limit = kWaitLimit;
+    if (const char *e = getenv("RS_DEBUG_WAIT_LIMIT")) {
+        const long long v = atoll(e);
+        if (v > 0) a.wait_limit = v;
+    }
     cudaStream_t st = (cudaStream_t)stream;
 
     // a map over an empty KV cache is never dereferenced: point it at q

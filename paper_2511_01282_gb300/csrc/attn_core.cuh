@@ -99,6 +99,7 @@ struct AttnArgs {
     CombJob *jobs;  // [gridDim.x]
     int2 *ranges;   // [gridDim.x]: each CTA's unit range [x, y)
     int kv_stream;  // the launch's K/V is large next to L2: stream tiles read once
+    long long wait_limit;  // clock cycles a pipeline wait may take before the CTA gives up
     int B, Hq, Hkv, D;
     float scale;
     float *out, *lse;
@@ -275,8 +276,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 // Warp-uniform bounded wait for the softmax warps: every lane waits, and the
 // warp gives up together if any lane gave up, so warp-wide instructions
 // (tcgen05.ld/st, vote) that follow always see the whole warp.
-__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
-    const bool ok = sm100::mbar_wait(bar, parity, abort, kWaitLimit);
+__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, volatile int *abort, long long limit) {
+    const bool ok = sm100::mbar_wait(bar, parity, abort, limit);
     return __all_sync(0xffffffffu, ok);
 }
 
@@ -365,14 +366,18 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                     unsigned char *sk = smem + kSmemK + st * kTileBytes;
                     unsigned char *sv = smem + kSmemV + st * kTileBytes;
                     // K is released as soon as S = Q K^T of the tile is done, V after P V
-                    if (!(ok = mbar_wait(&kempty[st], free_par, s_abort, kWaitLimit))) break;
+                    if (!(ok = mbar_wait(&kempty[st], free_par, s_abort, a.wait_limit))) break;
                     mbar_expect_tx(&kfull[st], kTileTx);
 #pragma unroll
                     for (int kb = 0; kb < kKB; ++kb) {
                         if (reread) tma_load_3d(sk + kb * 16384, &tmk, &kfull[st], kb * 64, pc.kvh, row);
                         else tma_load_3d_hint(sk + kb * 16384, &tmk, &kfull[st], kb * 64, pc.kvh, row, once);
                     }
-                    if (!(ok = mbar_wait(&vempty[st], free_par, s_abort, kWaitLimit))) break;
+                    if (!(ok = mbar_wait(&vempty[st], free_par, s_abort, a.wait_limit))) {
+                        volatile int no_abort = 0;  // this tile's K copy is in flight: let it land
+                        mbar_wait(&kfull[st], (uint32_t)((g / kNS) & 1), &no_abort, kWaitLimit);
+                        break;
+                    }
                     mbar_expect_tx(&vfull[st], kTileTx);
 #pragma unroll
                     for (int kb = 0; kb < kKB; ++kb) {
@@ -422,7 +427,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
             bool ok = true;
             auto issue_s = [&](long long gt) -> bool {
                 const int st = (int)(gt % kNS);
-                if (!mbar_wait(&kfull[st], (uint32_t)((gt / kNS) & 1), s_abort, kWaitLimit)) return false;
+                if (!mbar_wait(&kfull[st], (uint32_t)((gt / kNS) & 1), s_abort, a.wait_limit)) return false;
                 tc_fence_after();
                 const uint32_t k_addr = smem_u32(smem + kSmemK + st * kTileBytes);
                 const uint32_t d_s = tmem + kTmS + (uint32_t)(gt & 1) * 128;
@@ -437,17 +442,17 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
             for (long long u = u0; u < u1 && ok; ++piece) {
                 const Piece pc = piece_at(info, s_pref, a.B, u, u0, u1, c);
                 const int n = pc.j1 - pc.j0;
-                if (!(ok = mbar_wait(qready, (uint32_t)(piece & 1), s_abort, kWaitLimit))) break;
+                if (!(ok = mbar_wait(qready, (uint32_t)(piece & 1), s_abort, a.wait_limit))) break;
                 tc_fence_after();
                 if (!(ok = issue_s(g))) break;
                 for (int tl = 0; tl < n && ok; ++tl) {
                     const long long gt = g + tl;
                     if (tl + 1 < n && !(ok = issue_s(gt + 1))) break;
                     const int st = (int)(gt % kNS);
-                    if (!(ok = mbar_wait(&pfull[gt & 1], (uint32_t)((gt >> 1) & 1), s_abort, kWaitLimit))) break;
-                    if (!(ok = mbar_wait(&vfull[st], (uint32_t)((gt / kNS) & 1), s_abort, kWaitLimit))) break;
+                    if (!(ok = mbar_wait(&pfull[gt & 1], (uint32_t)((gt >> 1) & 1), s_abort, a.wait_limit))) break;
+                    if (!(ok = mbar_wait(&vfull[st], (uint32_t)((gt / kNS) & 1), s_abort, a.wait_limit))) break;
                     if (tl == 0 && piece > 0 &&
-                        !(ok = mbar_wait(ofree, (uint32_t)((piece - 1) & 1), s_abort, kWaitLimit)))
+                        !(ok = mbar_wait(ofree, (uint32_t)((piece - 1) & 1), s_abort, a.wait_limit)))
                         break;
                     tc_fence_after();
                     const uint32_t v_addr = smem_u32(smem + kSmemV + st * kTileBytes);
@@ -527,7 +532,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                 const long long gt = g + tl;
                 const int buf = (int)(gt & 1);
                 const int jt = pc.j0 + tl;
-                if (!(ok = warp_wait(&sfull[buf], (uint32_t)((gt >> 1) & 1), s_abort))) break;
+                if (!(ok = warp_wait(&sfull[buf], (uint32_t)((gt >> 1) & 1), s_abort, a.wait_limit))) break;
                 tc_fence_after();
                 // S of this tile is complete, so its K stage is free: released
                 // here rather than by a second commit on the MMA thread
@@ -569,7 +574,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                 // wait: a named barrier could not give up if a peer aborted)
                 s_mx[buf][hw][r] = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
                 warp_arrive(&mxready[buf]);
-                if (!(ok = warp_wait(&mxready[buf], (uint32_t)((gt >> 1) & 1), s_abort))) break;
+                if (!(ok = warp_wait(&mxready[buf], (uint32_t)((gt >> 1) & 1), s_abort, a.wait_limit))) break;
                 const float mt = fmaxf(s_mx[buf][0][r], s_mx[buf][1][r]) * cexp;
                 // lazy rescale: move the reference maximum only when it grows by
                 // more than 2^8; tcgen05.ld/st are warp-wide, so the O pass runs
@@ -578,7 +583,7 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
                 const float corr = grow ? ex2(m_used - mt) : 1.f;  // 0 when m_used is -inf
                 if (tl > 0 && __any_sync(0xffffffffu, grow)) {
                     const long long pv = gt - 1;  // O must hold PV of the previous tile
-                    if (!(ok = warp_wait(&vempty[(int)(pv % kNS)], (uint32_t)((pv / kNS) & 1), s_abort))) break;
+                    if (!(ok = warp_wait(&vempty[(int)(pv % kNS)], (uint32_t)((pv / kNS) & 1), s_abort, a.wait_limit))) break;
                     tc_fence_after();
 #pragma unroll
                     for (int ch = 0; ch < kHalfO / 32; ++ch) {
@@ -616,11 +621,11 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
             // epilogue: the row sum is the two warpgroups' partial sums
             s_l[hw][r] = l;
             warp_arrive(lready);
-            if (!(ok = warp_wait(lready, (uint32_t)(piece & 1), s_abort))) break;
+            if (!(ok = warp_wait(lready, (uint32_t)(piece & 1), s_abort, a.wait_limit))) break;
             const float lt = s_l[0][r] + s_l[1][r];
             {
                 const long long pv = g + n - 1;  // wait for PV of the last tile
-                if (!(ok = warp_wait(&vempty[(int)(pv % kNS)], (uint32_t)((pv / kNS) & 1), s_abort))) break;
+                if (!(ok = warp_wait(&vempty[(int)(pv % kNS)], (uint32_t)((pv / kNS) & 1), s_abort, a.wait_limit))) break;
             }
             tc_fence_after();
             const long long orow = (long long)(n0 + i) * a.Hq + h;

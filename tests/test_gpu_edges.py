@@ -91,6 +91,26 @@ def test_attention_many_requests(B, ctx_hi, D):
     assert np.abs(got - ref["out"].reshape(len(rows), D)).max() < 1e-2
 
 
+def test_attention_wait_time_out_reports_status_and_recovers(monkeypatch):
+    # every pipeline wait limited to 200 clock cycles: the first waits give
+    # up, the CTAs drain their copies and MMAs, free TMEM and flag the
+    # requests they held; the next call, with the normal limit, is correct
+    rng = np.random.default_rng(2)
+    Hq, Hkv, D = 4, 2, 128
+    trees = [[-1, 0, 0, 1], [-1] + [int(rng.integers(0, i)) for i in range(1, 40)]]
+    S = [700, 1500]
+    inp = _attn_inputs(rng, Hq, Hkv, D, S, trees)
+    monkeypatch.setenv("RS_DEBUG_WAIT_LIMIT", "200")
+    _, _, status = _run_attn(*inp, Hq, Hkv, D, D ** -0.5)
+    assert (status & rs.RS_ST_TIMEOUT).any()
+    monkeypatch.delenv("RS_DEBUG_WAIT_LIMIT")
+    out, lse, status = _run_attn(*inp, Hq, Hkv, D, D ** -0.5)
+    assert (status == 0).all()
+    q, k, v, kv_off, ctx, node_off, parents = inp
+    ref = oracle.tree_attn(q, k, v, kv_off, ctx, node_off, parents, Hq, Hkv, D, D ** -0.5)
+    assert np.abs(out.reshape(-1, D) - ref["out"]).max() < 1e-2
+
+
 def test_attention_single_node_and_tile_straddling_tree():
     rng = np.random.default_rng(1)
     Hq, Hkv, D = 6, 3, 64
