@@ -1,19 +1,21 @@
 // attn_core.cuh -- the tensor-core (tcgen05) core of rs_tree_verify_attn and
 // the shared work schedule.
 //
-// One CTA per SM walks its contiguous range of KV-tile units (see attn.cu).
+// One CTA per SM walks its contiguous range of KV-tile units (see attn.cu
+// and the Split below for how the ranges are cut).
 // Within a CTA, warps are specialised:
 //   warp 8 (1 thread)  TMA: K and V tiles of 128 keys x D into a 3-stage
 //                      ring of 128-byte-swizzled shared-memory buffers (a
-//                      K slot is refilled once S of its tile is done, a V slot
-//                      once P V is);
+//                      K slot is refilled once the softmax warps have seen S
+//                      of its tile complete, a V slot once P V is);
 //   warp 9 (1 thread)  MMA: S = Q K^T into one of two TMEM buffers, then
 //                      O += P V with P read from TMEM (bf16, written over
 //                      S by the softmax warps) and V from shared memory;
 //   warps 0-7          two softmax warpgroups over the same 128 rows (the
 //                      TMEM lane of a warp is fixed by warp % 4), each
 //                      taking 64 of a tile's 128 keys; they agree on the
-//                      row maxima through a named barrier.  Per row: Q into
+//                      row maxima through shared memory and an mbarrier.
+//                      Per row: Q into
 //                      TMEM, mask
 //                      (prefix always visible, tree slots by the ancestor
 //                      bit set, other requests' keys never), online softmax in
