@@ -103,12 +103,6 @@ __device__ __forceinline__ float warp_sum(float v) {
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     return v;
 }
-__device__ __forceinline__ int warp_sum_i(int v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    return v;
-}
-
 // (value, id) total order used for argmax / TopK: larger value first, then
 // smaller id.  Returns true when (va, ia) comes strictly before (vb, ib).
 __device__ __forceinline__ bool vi_before(float va, int ia, float vb, int ib) {
