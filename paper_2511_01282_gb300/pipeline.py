@@ -183,7 +183,10 @@ class VerifyStep:
 
     # ------------------------------------------------------ host round trip
     def upload(self, stream=None):
-        """Copy every input from pinned host memory: one async copy on `stream`."""
+        """Copy every input from pinned host memory: one async copy on `stream`
+        (needs VerifyStep(..., pinned_host=True) or a shared host_blob)."""
+        if self.pinned_blob is None:
+            raise RuntimeError("VerifyStep.upload: built without pinned_host=True")
         s = torch.cuda.current_stream() if stream is None else stream
         with torch.cuda.stream(s):
             self.dev_blob.copy_(self.pinned_blob, non_blocking=True)
