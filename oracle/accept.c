@@ -28,7 +28,11 @@
  *     fails the relaxed check; otherwise it counts the consecutive greedy
  *     matches xi that FOLLOW cur; if xi >= m the acceptance extends over the
  *     relaxed token and those matches (last = cur + 1 + xi, cur = last),
- *     else cur advances by one.  The accepted length is last;
+ *     else cur advances by one.  The accepted length is last.  This reading
+ *     is parity unpinned against the paper, which prints no worked example
+ *     of the procedure; the tests pin it to hand-worked cases of the reading
+ *     and to its closed special cases (phi = 0, beta = 1 or tau = 0 reduce
+ *     it to strict verification; an all-greedy chain is accepted whole);
  *   - the winner is the longest accepted path; ties go to the model tree,
  *     then to the chain that was selected first; all zero -> no winner;
  *   - the bonus token is the argmax of the last accepted node's row (the
