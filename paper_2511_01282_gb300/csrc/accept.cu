@@ -8,14 +8,20 @@
 // (logit desc, id asc); the top-beta is exact and sort-free apart from one
 // 16-lane sort that sets the candidate threshold.  No dynamic register
 // indexing.
-// Kernel 2 (accept_merge): one warp per row merges the chunk results into
-// argmax, top-beta, log-sum-exp, the row's largest logit (workspace, for
-// kernel 3) and (optionally) the row entropy.
+// Row merge: one warp per row merges the chunk results into argmax,
+// top-beta, log-sum-exp, the row's largest logit (workspace, for kernel 3)
+// and (optionally) the row entropy.  When a row has at most 8 chunks the
+// row's chunk CTAs form one cluster: each pushes its results into CTA 0's
+// shared memory and CTA 0 merges them after the cluster barrier, so the row
+// statistics need no second kernel.  Longer rows write their chunk results
+// to the workspace and kernel 2 (accept_merge) merges them.
 // Kernel 3 (accept_decide): one CTA per request checks the tree, verifies
 // model nodes (each thread walks its own root path over per-node match
 // flags), runs the look-ahead procedure per chain (one thread per chain),
 // picks the winner and updates the scores (one thread per selection).
 #include <math.h>
+
+#include <cooperative_groups.h>
 
 #include <algorithm>
 
@@ -25,11 +31,14 @@
 namespace rs {
 namespace {
 
+namespace cg = cooperative_groups;
+
 constexpr int kAccThreads = 256;
 constexpr int kAccVpt = 32;
 constexpr int kAccChunk = kAccThreads * kAccVpt;
 constexpr int kNoId = 0x7fffffff;  // "no candidate": after every real (v, id)
 constexpr int kCandCap = 64;        // per-warp candidate buffer (logits at or above the threshold)
+constexpr int kFuseMax = 8;         // rows of at most this many chunks merge inside their cluster
 
 struct VI {
     float v;
@@ -96,8 +105,59 @@ struct RowsShared {
     float hmax[kHalves];
     VI wtop[kAccThreads / 32][RS_MAX_BETA];  // per-warp lists (tie fallback)
     VI cbuf[kCandCap];                       // the chunk's candidates
+    VI rx_cand[kFuseMax * RS_MAX_BETA];      // CTA 0 of a row: every chunk's beta best
+    MS rx_ms[kFuseMax];                      // and every chunk's triple
     int cnt;
 };
+
+// Per-row outputs of the row statistics.
+struct RowOut {
+    int32_t *argmax, *topk;
+    float *lse, *entropy, *rowmax;  // entropy may be null
+};
+
+// One warp merges row r's chunk results: the chunk (m, s, w) triples into
+// the log-sum-exp (and the entropy), the chunk candidate lists (ncand <=
+// 32 kPer pairs, loaded once into registers) into argmax and top-beta by
+// beta rounds of a warp-wide "best after the previous winner" reduction.
+template <int kPer>
+__device__ __forceinline__ void merge_row(const VI *cand, int ncand, const MS *part, int nchunks, int beta,
+                                          long long r, const RowOut &o, int lane) {
+    MS ms{-INFINITY, 0.f, 0.f};
+    for (int c = lane; c < nchunks; c += 32) ms = ms_merge(ms, part[c]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) ms = ms_merge(ms, ms_shfl(ms, off));
+    VI cv[kPer];
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+        const int c = lane + 32 * q;
+        cv[q] = c < ncand ? cand[c] : VI{-INFINITY, kNoId};
+    }
+    VI prev{INFINITY, -1};
+    for (int k = 0; k < beta; ++k) {
+        VI best{-INFINITY, kNoId};
+#pragma unroll
+        for (int q = 0; q < kPer; ++q) {
+            const VI x = cv[q];
+            if (x.i != kNoId && vi_before(prev.v, prev.i, x.v, x.i) && vi_before(x.v, x.i, best.v, best.i))
+                best = x;
+        }
+        best = warp_vi_best(best);
+        prev = best;
+        if (lane == 0) {
+            const int id = best.i == kNoId ? -1 : best.i;
+            o.topk[r * beta + k] = id;
+            if (k == 0) {
+                o.argmax[r] = id;
+                o.rowmax[r] = best.v;
+            }
+        }
+    }
+    if (lane == 0) {
+        o.lse[r] = ms.s > 0.f ? ms.m + __logf(ms.s) : -INFINITY;
+        if (o.entropy) o.entropy[r] = ms.s > 0.f ? (__logf(ms.s) - ms.w / ms.s) : 0.f;
+    }
+}
 
 // One CTA per (row, 8192-logit chunk) item: the chunk's (max, sum e^(z -
 // max)[, sum e^(z - max) (z - max)]) triple and its beta best (logit, id)
@@ -115,19 +175,36 @@ struct RowsShared {
 //     candidates before it in the total order).  If ties at T overflow the
 //     buffer, every warp ranks its own logits by beta "best after the
 //     previous winner" rounds and warp 0 merges the eight lists (exact too).
-template <bool kVec, bool kEnt>
+//   * kFuse: the chunk's results go to CTA 0 of the row (the CTAs of a row
+//     are one cluster, chunk = rank), which merges the row after the
+//     cluster barrier; otherwise they go to the workspace for accept_merge.
+template <bool kVec, bool kEnt, bool kFuse>
 __global__ void __launch_bounds__(kAccThreads, 4)
 accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *__restrict__ cand,
-            MS *__restrict__ part) {
+            MS *__restrict__ part, RowOut o) {
     pdl_enter();
     __shared__ RowsShared sh;
     const long long blk = blockIdx.x;
     const long long r = blockIdx.x / (unsigned)nchunks;  // 32-bit division
-    const int c0 = (int)(blk - r * nchunks) * kAccChunk;
+    const int chunk = (int)(blk - r * nchunks);
+    const int c0 = chunk * kAccChunk;
     const float *row = logits + r * (long long)V;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     constexpr float kL2E = 1.4426950408889634f;
+    const bool clustered = kFuse && nchunks > 1;
+    if (clustered) cluster_arrive_relaxed();
     if (tid == 0) sh.cnt = 0;
+    VI *dcand = cand + blk * beta;  // where this chunk's beta best and triple go
+    MS *dms = part + blk;
+    if (kFuse) {
+        dcand = &sh.rx_cand[chunk * beta];
+        dms = &sh.rx_ms[chunk];
+        if (clustered) {
+            cg::cluster_group cl = cg::this_cluster();
+            dcand = cl.map_shared_rank(dcand, 0);
+            dms = cl.map_shared_rank(dms, 0);
+        }
+    }
 
     // logit id of register j (ids >= V are padding, held as -inf)
     auto id_of = [&](int j) -> int {
@@ -216,6 +293,7 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
     }
     __syncthreads();
     const int total = sh.cnt;
+    if (clustered) cluster_wait();  // every CTA of the row runs: CTA 0's shared memory is live
     if (total <= kCandCap) {
         if (warp == 0) {
             VI x0 = lane < total ? sh.cbuf[lane] : VI{-INFINITY, kNoId};
@@ -226,9 +304,9 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
                 r0 += vi_before(y.v, y.i, x0.v, x0.i);
                 r1 += vi_before(y.v, y.i, x1.v, x1.i);
             }
-            if (lane < total && r0 < beta) cand[blk * beta + r0] = x0;
-            if (lane + 32 < total && r1 < beta) cand[blk * beta + r1] = x1;
-            if (lane >= total && lane < beta) cand[blk * beta + lane] = VI{-INFINITY, kNoId};
+            if (lane < total && r0 < beta) dcand[r0] = x0;
+            if (lane + 32 < total && r1 < beta) dcand[r1] = x1;
+            if (lane >= total && lane < beta) dcand[lane] = VI{-INFINITY, kNoId};
         }
     } else {
         VI prev{INFINITY, -1};
@@ -258,7 +336,7 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
                 }
                 best = warp_vi_best(best);
                 prevb = best;
-                if (lane == 0) cand[blk * beta + k] = best;
+                if (lane == 0) dcand[k] = best;
             }
         }
     }
@@ -266,60 +344,33 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
         MS a = lane < kAccThreads / 32 ? sh.sms[lane] : MS{-INFINITY, 0.f, 0.f};
 #pragma unroll
         for (int o = 4; o > 0; o >>= 1) a = ms_merge(a, ms_shfl(a, o));
-        if (lane == 0) part[blk] = a;
+        if (lane == 0) *dms = a;
+    }
+    if (kFuse) {
+        if (clustered) {
+            cluster_arrive_release();  // the pushes above are visible in CTA 0 after the wait
+            cluster_wait();
+        } else {
+            __syncthreads();
+        }
+        if (chunk == 0 && warp == 0)
+            merge_row<kFuseMax * RS_MAX_BETA / 32>(sh.rx_cand, nchunks * beta, sh.rx_ms, nchunks, beta, r, o, lane);
     }
 }
 
-// Row statistics: one warp per row merges the chunk candidates (loaded
-// once into registers, <= 32 * kCandPerLane) by beta rounds of a warp-wide
-// "best after the previous winner" reduction, and the chunk (m, s, w)
-// triples into the log-sum-exp (and the entropy when asked).
+// Row statistics of rows longer than kFuseMax chunks: one warp per row
+// merges the chunk results from the workspace.
 constexpr int kMergeThreads = 256;
 constexpr int kCandPerLane = 8;
 
 __global__ void __launch_bounds__(kMergeThreads)
-accept_merge(const VI *__restrict__ cand, const MS *__restrict__ part, int nchunks, int beta, int R,
-             int32_t *__restrict__ argmax, int32_t *__restrict__ topk, float *__restrict__ lse,
-             float *__restrict__ entropy, float *__restrict__ rowmax) {
+accept_merge(const VI *__restrict__ cand, const MS *__restrict__ part, int nchunks, int beta, int R, RowOut o) {
     pdl_enter();
     const int lane = threadIdx.x & 31;
     const long long r = (long long)blockIdx.x * (kMergeThreads / 32) + (threadIdx.x >> 5);
     if (r >= R) return;
-    MS ms{-INFINITY, 0.f, 0.f};
-    for (int c = lane; c < nchunks; c += 32) ms = ms_merge(ms, part[r * nchunks + c]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) ms = ms_merge(ms, ms_shfl(ms, o));
     const int ncand = nchunks * beta;
-    VI cv[kCandPerLane];
-#pragma unroll
-    for (int q = 0; q < kCandPerLane; ++q) {
-        const int c = lane + 32 * q;
-        cv[q] = c < ncand ? cand[r * ncand + c] : VI{-INFINITY, kNoId};
-    }
-    VI prev{INFINITY, -1};
-    for (int k = 0; k < beta; ++k) {
-        VI best{-INFINITY, kNoId};
-#pragma unroll
-        for (int q = 0; q < kCandPerLane; ++q) {
-            const VI x = cv[q];
-            if (x.i != kNoId && vi_before(prev.v, prev.i, x.v, x.i) && vi_before(x.v, x.i, best.v, best.i))
-                best = x;
-        }
-        best = warp_vi_best(best);
-        prev = best;
-        if (lane == 0) {
-            const int id = best.i == kNoId ? -1 : best.i;
-            topk[r * beta + k] = id;
-            if (k == 0) {
-                argmax[r] = id;
-                rowmax[r] = best.v;
-            }
-        }
-    }
-    if (lane == 0) {
-        lse[r] = ms.s > 0.f ? ms.m + __logf(ms.s) : -INFINITY;
-        if (entropy) entropy[r] = ms.s > 0.f ? (__logf(ms.s) - ms.w / ms.s) : 0.f;
-    }
+    merge_row<kCandPerLane>(cand + r * ncand, ncand, part + r * nchunks, nchunks, beta, r, o, lane);
 }
 
 constexpr int kDecThreads = 512;
@@ -601,6 +652,15 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
 
 using namespace rs;
 
+namespace {
+using RowsFn = void (*)(const float *, int, int, int, VI *, MS *, RowOut);
+template <bool kFuse>
+RowsFn rows_fn(bool vec, bool ent) {
+    if (vec) return ent ? accept_rows<true, true, kFuse> : accept_rows<true, false, kFuse>;
+    return ent ? accept_rows<false, true, kFuse> : accept_rows<false, false, kFuse>;
+}
+}  // namespace
+
 extern "C" size_t rs_accept_workspace_size(int R, int V, int beta) {
     if (R < 0 || V < 1 || beta < 1) return 0;
     int nchunks = (V + kAccChunk - 1) / kAccChunk;
@@ -656,20 +716,20 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
         RS_CHECK_ARG(blocks < (1ll << 30), "rs_accept: R*chunks too large");
         const bool vec = (V % 4 == 0) && (((uintptr_t)logits & 15) == 0);
         const bool ent = entropy != nullptr;
+        const bool fuse = nchunks <= kFuseMax;
+        const RowOut ro{argmax, topk, lse, entropy, rowmax};
+        const RowsFn fn = fuse ? rows_fn<true>(vec, ent) : rows_fn<false>(vec, ent);
         const dim3 grid((unsigned)blocks);
-        if (vec && ent)
-            launch_pdl(accept_rows<true, true>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand, part);
-        else if (vec)
-            launch_pdl(accept_rows<true, false>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand, part);
-        else if (ent)
-            launch_pdl(accept_rows<false, true>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand, part);
+        if (fuse && nchunks > 1)
+            launch_pdl_cluster(fn, grid, dim3(kAccThreads), 0, st, nchunks, logits, V, nchunks, p.beta, cand, part, ro);
         else
-            launch_pdl(accept_rows<false, false>, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand,
-                part);
+            launch_pdl(fn, grid, dim3(kAccThreads), 0, st, logits, V, nchunks, p.beta, cand, part, ro);
         RS_CHECK_LAUNCH("rs_accept/accept_rows");
-        launch_pdl(accept_merge, dim3((R + kMergeThreads / 32 - 1) / (kMergeThreads / 32)), dim3(kMergeThreads),
-            0, st, cand, part, nchunks, p.beta, R, argmax, topk, lse, entropy, rowmax);
-        RS_CHECK_LAUNCH("rs_accept/accept_merge");
+        if (!fuse) {
+            launch_pdl(accept_merge, dim3((R + kMergeThreads / 32 - 1) / (kMergeThreads / 32)), dim3(kMergeThreads),
+                0, st, cand, part, nchunks, p.beta, R, ro);
+            RS_CHECK_LAUNCH("rs_accept/accept_merge");
+        }
     }
     if (B > 0) {
         launch_pdl(accept_decide, dim3(B), dim3(kDecThreads), 0, st, logits, V, node_off, tokens, parents,

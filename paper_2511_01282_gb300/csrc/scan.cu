@@ -17,8 +17,8 @@
 // match than the buffer holds, per-thread lists merged block-wide are used
 // instead.  In the split case every CTA pushes its count
 // to all peers and its best top_c to CTA 0 through distributed shared memory
-// before one cluster barrier; after it nobody touches another CTA's shared
-// memory.  CTA 0 ranks the (at most 64) listed matches the same way and
+// (once the cluster barrier's entry phase shows every CTA running) before one
+// cluster barrier; after it nobody touches another CTA's shared memory.  CTA 0 ranks the (at most 64) listed matches the same way and
 // gathers the selected continuations (from the staged window when it alone
 // scanned the buffer).  A slice that
 // spans several windows stages them in turn, and again for the position pass.
@@ -224,6 +224,7 @@ match_scan_kernel(const int32_t *__restrict__ tokens, const int64_t *__restrict_
     // t <= kWin: the tokens [0, t) all fit the staged window (after the halo)
     const bool solo = !run || t <= kWin;  // CTA 0 alone, no cluster barrier
     if (solo && crank != 0) return;
+    if (!solo) cluster_arrive_relaxed();  // this CTA runs; the wait sits before the first push
     long long lo = 0, hi = 0;
     if (run) {
         const long long n = t - 1;
@@ -338,13 +339,15 @@ match_scan_kernel(const int32_t *__restrict__ tokens, const int64_t *__restrict_
     long long offset = 0, total = cta_total;
     if (!solo) {
         __syncthreads();  // this CTA's top list is complete
+        cluster_wait();   // every CTA of the cluster is running
         if (tid < kScanCluster) *cluster.map_shared_rank(&sh.peer_cnt[crank], tid) = cta_total;
         if (tid < RS_MAX_TOPC) {
             *cluster.map_shared_rank(&sh.peer_s[crank][tid], 0) = sh.top_s[tid];
             *cluster.map_shared_rank(&sh.peer_p[crank][tid], 0) = sh.top_p[tid];
         }
         if (tid == 0) *cluster.map_shared_rank(&sh.peer_n[crank], 0) = sh.ntop;
-        cluster.sync();  // the only cluster barrier: every push is visible after it
+        cluster_arrive_release();  // every push is visible after the wait
+        cluster_wait();
         total = 0;
         for (int r = 0; r < kScanCluster; ++r) {
             const long long c = sh.peer_cnt[r];
