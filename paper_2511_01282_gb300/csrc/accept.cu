@@ -239,7 +239,7 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
     const float mx = fmaxf(fmaxf(fmaxf(g[0], g[1]), fmaxf(g[2], g[3])), fmaxf(fmaxf(g[4], g[5]), fmaxf(g[6], g[7])));
     float hm = mx;
 #pragma unroll
-    for (int o = 1; o < 16; o <<= 1) hm = fmaxf(hm, __shfl_xor_sync(0xffffffffu, hm, o));
+    for (int off = 1; off < 16; off <<= 1) hm = fmaxf(hm, __shfl_xor_sync(0xffffffffu, hm, off));
     const float wmax = fmaxf(hm, __shfl_xor_sync(0xffffffffu, hm, 16));
     if ((lane & 15) == 0) sh.hmax[2 * warp + (lane >> 4)] = hm;
 
@@ -263,9 +263,9 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
         float ss = (s4[0] + s4[1]) + (s4[2] + s4[3]);
         float ww = (w4[0] + w4[1]) + (w4[2] + w4[3]);
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            ss += __shfl_xor_sync(0xffffffffu, ss, o);
-            if (kEnt) ww += __shfl_xor_sync(0xffffffffu, ww, o);
+        for (int off = 16; off > 0; off >>= 1) {
+            ss += __shfl_xor_sync(0xffffffffu, ss, off);
+            if (kEnt) ww += __shfl_xor_sync(0xffffffffu, ww, off);
         }
         t.s = ss;
         t.w = ww * 0.6931471805599453f;
@@ -343,7 +343,7 @@ accept_rows(const float *__restrict__ logits, int V, int nchunks, int beta, VI *
     if (warp == 0) {  // the eight warp triples, merged as a 3-level tree
         MS a = lane < kAccThreads / 32 ? sh.sms[lane] : MS{-INFINITY, 0.f, 0.f};
 #pragma unroll
-        for (int o = 4; o > 0; o >>= 1) a = ms_merge(a, ms_shfl(a, o));
+        for (int off = 4; off > 0; off >>= 1) a = ms_merge(a, ms_shfl(a, off));
         if (lane == 0) *dms = a;
     }
     if (kFuse) {
