@@ -5,10 +5,10 @@
  *
  * One decoding step of Algorithm 1, as four calls:
  *
- *   rs_entropy_gate     Section 3.2.1, Eq. 1-3 and step 4 (Alg. 1 step 1)
- *   rs_match_scan       Section 3.3 retrieval + selection   (Alg. 1 l.9-11)
- *   rs_tree_verify_attn tree attention of the verify pass   (Alg. 1 l.13/25)
- *   rs_accept           Section 3.4 verification, Eq. 4-5  (Alg. 1 l.13-22)
+ *   rs_entropy_gate     Section 3.2.1, Eq. 1-3, trigger decision (Alg. 1 triggering)
+ *   rs_match_scan       Section 3.3 retrieval + selection   (Alg. 1 retrieval)
+ *   rs_tree_verify_attn tree attention of the verify pass   (Alg. 1 verification)
+ *   rs_accept           Section 3.4 verification, Eq. 4-5  (Alg. 1 verify + EMA)
  *
  * General rules (every entry point):
  *   - All array arguments are DEVICE pointers owned by the caller, unless a
@@ -70,14 +70,14 @@ typedef enum {
                                for tests); the request's outputs are invalid   */
 
 /* -------------------------------------------------------------- parameters */
-/* Hyper-parameters of Algorithm 1 (Require line), Eq. 6-7 and Section 3.4.
+/* Hyper-parameters of Algorithm 1 (its inputs), Eq. 6-7 and Section 3.4.
  * Passed by value.  Defaults used by this project where the paper gives no
  * value: lambda_e 0.5, alpha 0.3, theta_score 0.3, beta 5, tau 3, phi 2,
  * m 2; the paper fixes theta_entropy = 1.5, top_c = 3 and l = 3. */
 typedef struct {
     int   l;              /* maximum key length, 1..RS_MAX_L                       */
     float lambda_e;       /* Eq. 2 length penalty                                  */
-    float theta_entropy;  /* step 4 trigger threshold, nats                        */
+    float theta_entropy;  /* trigger threshold of Section 3.2.1, nats              */
     float alpha;          /* Eq. 4 EMA rate, in [0, 1]                             */
     float theta_score;    /* Section 3.3 score threshold                           */
     int   top_c;          /* candidates kept, 1..RS_MAX_TOPC                       */
@@ -99,8 +99,8 @@ uint64_t rs_launch_count(void);
 
 /* ===================================================== rs_entropy_gate ====
  * Section 3.2.1 (Eq. 1: mean predictive entropy of a key; Eq. 2: C_k =
- * H_k + lambda_e / k; Eq. 3: k* = argmin C_k; step 4: trigger iff
- * H_{k*} <= theta_entropy), evaluated as Algorithm 1 step 1 does (k upward,
+ * H_k + lambda_e / k; Eq. 3: k* = argmin C_k; trigger decision: iff
+ * H_{k*} <= theta_entropy), evaluated as Algorithm 1's triggering does (k upward,
  * strict '<', so ties keep the shorter key).
  *
  *   logits     [R, V] fp32 row-major: the verify pass's next-token logits,
@@ -129,7 +129,7 @@ rs_status rs_entropy_gate(const float *logits, int R, int V, const int32_t *row_
                           void *workspace, size_t workspace_bytes, void *stream);
 
 /* ================================================ rs_entropy_gate_rows ====
- * The trigger of rs_entropy_gate (history push, H_k, C_k, k*, step 4) from
+ * The trigger of rs_entropy_gate (history push, H_k, C_k, k*, decision) from
  * row entropies computed elsewhere -- rs_accept's `entropy` output over the
  * same logits -- instead of from the logits.  Arguments as rs_entropy_gate;
  * `entropy` is an input here.  One kernel, no workspace.
@@ -165,7 +165,7 @@ rs_status rs_entropy_gate_noalloc(const float *logits, int R, int V, const int32
                                   void *stream);
 
 /* ======================================================= rs_match_scan ====
- * Section 3.3 "Selection Algorithm" and Algorithm 1 l.9-11: find every
+ * Section 3.3 "Selection Algorithm" and Algorithm 1's retrieval: find every
  * earlier occurrence of the key (the buffer's last k = k_star[b] tokens),
  * drop positions whose score is below theta_score, keep the top_c best by
  * score and gather their continuations.
@@ -177,7 +177,7 @@ rs_status rs_entropy_gate_noalloc(const float *logits, int R, int V, const int32
  *   k_star   [B] int32 key lengths (rs_entropy_gate's output); k <= 0 skips
  *            the request, k > RS_MAX_L skips it with RS_ST_TOO_LARGE.
  *   gate_ok  [B] uint8 or NULL: when given, requests with gate_ok[b] == 0
- *            are skipped (Algorithm 1 l.9 fires only when the entropy half
+ *            are skipped (Algorithm 1 retrieves only when the entropy half
  *            of the trigger holds).
  *   scores   [sum t_b] fp32 feedback scores, parallel to tokens (score of a
  *            match = score of its end position; initialise to S0 = 0.5).
@@ -204,8 +204,8 @@ rs_status rs_match_scan(const int32_t *tokens, const int64_t *tok_off, int B,
                         void *stream);
 
 /* ================================================= rs_tree_verify_attn ====
- * Attention of the verify pass over the packed draft tree (Algorithm 1
- * l.13 / l.25; the paper's "parallel verification", Section 3.3): every
+ * Attention of the verify pass over the packed draft tree (the verify
+ * forward of Algorithm 1; the paper's "parallel verification", Section 3.3): every
  * tree node attends to its request's whole committed prefix and to the
  * tree slots of its ancestors and itself.
  *
@@ -236,7 +236,7 @@ rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, const uint16
 
 /* =========================================================== rs_accept ====
  * Section 3.4 source-aware verification, the longest accepted path of
- * Algorithm 1 l.13 and the EMA feedback of Eq. 4-5 (Algorithm 1 l.15-22).
+ * Algorithm 1 and the EMA feedback of Eq. 4-5 (Algorithm 1's score update).
  *
  *   logits   [R, V] fp32 verify logits (row of node i predicts its children).
  *   node_off [B+1] int32;  tokens [R] int32 draft token of every node, in

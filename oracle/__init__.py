@@ -79,7 +79,7 @@ def entropy_rows(logits):
 
 
 def gate(H, row_off, row_commit, hist, hist_n, l, lambda_e, theta):
-    """Section 3.2.1 steps 1-4 (Algorithm 1 step 1) on given row entropies.
+    """Section 3.2.1 (entropy, confidence score, key selection, trigger decision; Algorithm 1's triggering) on given row entropies.
 
     ``hist`` [B, l] (oldest first) and ``hist_n`` [B] are copied, updated and
     returned; the inputs are left untouched.
@@ -101,7 +101,7 @@ def gate(H, row_off, row_commit, hist, hist_n, l, lambda_e, theta):
 # ---------------------------------------------------------------- match scan
 def match_scan(tokens, tok_off, k_star, scores, theta_score, top_c, span_len, pos_cap,
                gate_ok=None):
-    """Section 3.3 retrieval + selection (Algorithm 1 l.9-11)."""
+    """Section 3.3 retrieval + selection (Algorithm 1's retrieval)."""
     tokens = _c(tokens, np.int32)
     tok_off = _c(tok_off, np.int64)
     k_star = _c(k_star, np.int32)

@@ -11,9 +11,9 @@
  *     relaxed verification of retrieved drafts (Eq. 6: the token is among the
  *     beta most likely tokens; Eq. 7: log p(x1) - log p(x~) <= tau) and the
  *     look-ahead tolerance procedure;
- *   - Algorithm 1 l.13: the longest accepted path over all branches gives
+ *   - Algorithm 1 (verification): the longest accepted path over all branches gives
  *     X_accepted and the winning position;
- *   - Eq. 4-5 and Algorithm 1 l.15-22: S_p <- (1-alpha) S_p + alpha R_p with
+ *   - Eq. 4-5 and Algorithm 1's score update: S_p <- (1-alpha) S_p + alpha R_p with
  *     R_p = L_accepted / L_draft for the winner and 0 for every other
  *     selected position.
  *

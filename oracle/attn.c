@@ -4,7 +4,7 @@
  * TEST INFRASTRUCTURE ONLY (see rsref.h).
  *
  * The paper verifies the packed draft tree with one target forward
- * ("parallel verification", Section 3.3; Algorithm 1 l.13 and l.25) but does
+ * ("parallel verification", Section 3.3; both verifications of Algorithm 1) but does
  * not spell out the attention.  The standard reading is used: each tree node
  * attends to the whole committed prefix and to the tree slots of its
  * ancestors and itself (the draft tokens on its own root-to-node path), with

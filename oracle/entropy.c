@@ -5,8 +5,9 @@
  *
  * Follows Section 3.2.1: Eq. 1 (mean predictive entropy of a suffix key),
  * Eq. 2 (confidence score C_k = H_k + lambda_e / k), Eq. 3 (k* = argmin C_k)
- * and step 4 (trigger iff H_{k*} <= theta_entropy), in the order Algorithm 1
- * (step 1) evaluates them: k runs upward from 1 and a later k replaces the
+ * and the trigger decision (trigger iff H_{k*} <= theta_entropy), in the
+ * order Algorithm 1's entropy-guided triggering evaluates them: k runs
+ * upward from 1 and a later k replaces the
  * current best only when its C_k is strictly smaller.
  */
 #include <math.h>
@@ -39,7 +40,8 @@ void rsref_entropy_rows(const float *logits, long R, long V, double *H)
     for (long r = 0; r < R; ++r) H[r] = rsref_row_entropy(logits + r * V, V);
 }
 
-/* Section 3.2.1 steps 1-4 over the per-request entropy history.
+/* Section 3.2.1 (entropy, confidence score, key selection, trigger decision)
+ * over the per-request entropy history.
  * The history holds one entropy per committed token: the entropy of the
  * distribution that predicted it (the verify step's root row and the rows
  * of its accepted nodes), oldest first. */
@@ -66,7 +68,7 @@ void rsref_gate(const double *H, const long *row_off, const unsigned char *row_c
         }
         hist_n[b] = n;
 
-        /* Algorithm 1, step 1 */
+        /* Algorithm 1, entropy-guided triggering */
         double c_min = INFINITY, best = INFINITY;
         int kbest = 0;
         int kmax = n < l ? n : l;
@@ -84,6 +86,6 @@ void rsref_gate(const double *H, const long *row_off, const unsigned char *row_c
         }
         k_star[b] = kbest;
         h_best[b] = best;
-        ok[b] = (unsigned char)(kbest > 0 && best <= theta); /* step 4 */
+        ok[b] = (unsigned char)(kbest > 0 && best <= theta); /* trigger decision */
     }
 }

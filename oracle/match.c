@@ -5,7 +5,7 @@
  *
  * Follows Section 3.3 ("Selection Algorithm": retrieve every match position
  * of the key, drop those whose score is below theta_score, keep the top
- * candidates by score) and Algorithm 1 step 2 (Contains / RetrievePositions /
+ * candidates by score) and Algorithm 1's retrieval (Contains / RetrievePositions /
  * quality filter S_p >= theta_score / SelectTopK).  The suffix automaton of
  * the paper is an index over the same position set; here the set is found by
  * comparing the key with every window of the buffer.
@@ -72,7 +72,7 @@ int rsref_match_scan(const int *tokens, const long *tok_off, int B,
             if (!match) continue;
             if (cnt < pos_cap) pos[(long)b * pos_cap + cnt] = (int)p;
             ++cnt;
-            if ((double)S[p] >= theta_score) { /* quality filter (Alg. 1 l.11) */
+            if ((double)S[p] >= theta_score) { /* quality filter (Algorithm 1) */
                 cand[nf].s = S[p];
                 cand[nf].p = (int)p;
                 ++nf;

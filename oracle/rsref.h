@@ -42,7 +42,7 @@ double rsref_row_entropy(const float *z, long V);
 /* H[r] = rsref_row_entropy(logits + r*V, V) for r < R. */
 void rsref_entropy_rows(const float *logits, long R, long V, double *H);
 
-/* ---- Section 3.2.1 steps 1-4, Eq. 1-3; Algorithm 1 step 1 ------------- */
+/* ---- Section 3.2.1, Eq. 1-3; Algorithm 1's entropy-guided triggering -- */
 /* Pushes the entropies of the committed rows (row_commit[r] != 0, in row
  * order) of each request into its history (hist[b*l .. b*l+l-1], oldest
  * first, hist_n[b] valid entries, the newest at index hist_n[b]-1), then
@@ -55,7 +55,7 @@ void rsref_gate(const double *H, const long *row_off, const unsigned char *row_c
                 double *hist, int *hist_n,
                 int *k_star, double *h_best, unsigned char *ok);
 
-/* ---- Section 3.3 (retrieval, filtering, top-3); Alg. 1 l.9-11 --------- */
+/* ---- Section 3.3 (retrieval, filtering, top-3); Algorithm 1 retrieval -- */
 /* For request b with key length k = k_star[b] (skipped when k <= 0, or when
  * gate_ok is given and gate_ok[b] == 0): every buffer index p with
  * k-1 <= p <= t-2 whose trailing k tokens equal the buffer's last k tokens,
@@ -71,7 +71,7 @@ int rsref_match_scan(const int *tokens, const long *tok_off, int B,
                      int *count, int *pos, int *sel_pos, int *sel_len,
                      int *spans, int *n_sel, int *status);
 
-/* ---- Tree-verification attention (Alg. 1 l.13 "RelaxedVerify" forward) -- */
+/* ---- Tree-verification attention (the verify forward of Algorithm 1) -- */
 /* For each requested (global node r, q-head h): request b owns r; the keys
  * are every prefix slot j < ctx_len[b] and the tree slot ctx_len[b]+a of
  * every ancestor-or-self a of the node; K/V rows live at kv_off[b] + slot.
@@ -85,7 +85,7 @@ int rsref_tree_attn(const unsigned short *q, const unsigned short *k,
                     double scale, long n_rows, const long *row_node,
                     const int *row_head, double *out, double *lse);
 
-/* ---- Section 3.4 (Eq. 6-7, look-ahead tolerance), Eq. 4-5, Alg. 1 l.13-22 */
+/* ---- Section 3.4 (Eq. 6-7, look-ahead tolerance), Eq. 4-5, Algorithm 1 */
 /* Row statistics for every node row, then per request: strict acceptance of
  * model drafts, relaxed acceptance with look-ahead for retrieved chains,
  * longest accepted path, winner, bonus token, commit flags and the EMA

@@ -1,6 +1,6 @@
 // accept.cu -- rs_accept: source-aware verification (Section 3.4, Eq. 6-7
 // and the look-ahead tolerance procedure), longest accepted path and winner
-// (Algorithm 1 l.13), EMA feedback (Eq. 4-5, Algorithm 1 l.15-22).
+// (Algorithm 1), EMA feedback (Eq. 4-5 and Algorithm 1's score update).
 //
 // Kernel 1 (accept_rows): one CTA per (row, 8192-logit chunk) streams the
 // chunk once and produces its (max, sum e^(z - max)[, sum e^(z - max)

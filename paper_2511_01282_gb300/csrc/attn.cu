@@ -1,5 +1,5 @@
 // attn.cu -- rs_tree_verify_attn: attention of the verify pass over the
-// packed draft tree (Algorithm 1 l.13 / l.25; "parallel verification" of
+// packed draft tree (the verify forward of Algorithm 1; "parallel verification" of
 // Section 3.3).  Node i of request b attends to b's committed prefix and to
 // the tree slots of its ancestors and itself.
 //

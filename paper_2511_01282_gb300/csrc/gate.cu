@@ -1,5 +1,5 @@
 // gate.cu -- rs_entropy_gate: entropy-guided adaptive trigger
-// (Section 3.2.1, Eq. 1-3 and step 4; Algorithm 1 step 1).
+// (Section 3.2.1, Eq. 1-3 and the trigger decision; Algorithm 1's triggering).
 //
 // Kernel 1 (entropy_partial): one CTA per (row, 8192-logit chunk).  Each
 // thread streams 32 logits with 128-bit loads; relative to its warp's
@@ -164,7 +164,7 @@ entropy_merge(const Ent3 *__restrict__ part, int nchunks, int R, float *__restri
 // Per request: the committed rows' entropies, in row order, extend the
 // history and the newest l entries are kept; a block scan gives every
 // committed row its rank, so each surviving entry is written by its own
-// thread.  Then Algorithm 1 step 1 in fp64 with one lane per k (H_k, C_k)
+// thread.  Then Algorithm 1's triggering in fp64 with one lane per k (H_k, C_k)
 // and a warp argmin that keeps the smallest k among equal C_k (the first
 // strict minimum of the upward scan).
 constexpr int kPushThreads = 256;

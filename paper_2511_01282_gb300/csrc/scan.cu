@@ -1,5 +1,5 @@
 // scan.cu -- rs_match_scan: retrieval and feedback-driven candidate
-// selection (Section 3.3 "Selection Algorithm"; Algorithm 1 l.9-11).
+// selection (Section 3.3 "Selection Algorithm"; Algorithm 1's retrieval).
 //
 // One cluster of 8 CTAs (256 threads each) per request.  A buffer whose
 // candidate positions [0, t-2] fit one window of 8192 is handled by CTA 0

@@ -1,7 +1,7 @@
 """Pins for the oracle's verification, path selection and EMA update.
 
-Section 3.4 (Eq. 6-7, look-ahead tolerance), Eq. 4-5 and Algorithm 1
-l.13-22.  Checked against hand-worked look-ahead cases
+Section 3.4 (Eq. 6-7, look-ahead tolerance), Eq. 4-5 and Algorithm 1's
+verification and score update.  Checked against hand-worked look-ahead cases
 (tests/golden/lookahead_cases.json), numpy's lexicographic sort and scipy's
 log-softmax for the row statistics, brute-force path enumeration for the
 model tree, the reductions the definition implies (phi = 0 or beta = 1 is
