@@ -438,7 +438,7 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
     }
     __syncthreads();
 
-    // ---- round 1 + 2: tree, row statistics, token logits ----
+    // ---- the two dependent read rounds: tree and row statistics, then token logits ----
     if (st == 0) {
         for (int i = tid; i < N; i += kDecThreads) {
             const int pa = parents[n0 + i];
