@@ -149,10 +149,12 @@ def test_unaligned_and_odd_logits():
     check_accept(w, st)
 
 
-@pytest.mark.parametrize("V,beta", [(8193, 5), (20003, 16), (65536, 16), (65537, 16), (70000, 5)])
+@pytest.mark.parametrize("V,beta", [(8193, 5), (20003, 16), (65536, 16), (65537, 16), (70000, 5),
+                                    (100000, 16), (131072, 5), (131073, 5)])
 def test_accept_chunk_counts(V, beta):
     # rows of 2 to 8 chunks of 8192 logits are merged inside their cluster,
-    # longer rows by the separate merge kernel; V % 4 != 0 takes scalar loads
+    # longer rows (9 to 17 chunks here) by the separate merge kernel, up to
+    # its 256 candidates a row; V % 4 != 0 takes scalar loads
     w = synth.build(synth.small_spec(B=2, V=V, beta=beta), seed=V % 97)
     st = make_step(w)
     check_accept(w, st)
