@@ -209,10 +209,40 @@ class VerifyStep:
         return {k: torch.empty(self.out[k].shape, dtype=self.out[k].dtype).pin_memory()
                 for k in self.RESULT_KEYS}
 
+    # ------------------------------------------- state carried across steps
+    STATE_KEYS = ("hist", "hist_n", "scores")
+
     def reset_state(self):
         """Restore the in/out state (history, scores) to the host inputs."""
-        for k in ("hist", "hist_n", "scores"):
+        for k in self.STATE_KEYS:
             self.d[k].copy_(torch.from_numpy(self.host[k]))
+
+    def state(self):
+        """Checkpoint of the feedback state the decoding loop carries from step
+        to step: the entropy history of the trigger (Section 3.2.1) and the EMA
+        score table of the selection (Eq. 4-5), as host arrays.  Synchronise
+        the stream the steps ran on first."""
+        return {k: self.d[k].cpu().numpy().copy() for k in self.STATE_KEYS}
+
+    def load_state(self, state):
+        """Resume from a checkpoint taken by state() on a batch of the same
+        shapes (history [B, l], counts [B], scores parallel to the tokens)."""
+        for k in self.STATE_KEYS:
+            a = np.asarray(state[k])
+            ref = self.host[k]
+            if a.shape != ref.shape or a.dtype != ref.dtype:
+                raise ValueError("VerifyStep.load_state: %s is %s %s, this batch needs %s %s"
+                                 % (k, a.dtype, a.shape, ref.dtype, ref.shape))
+        for k in self.STATE_KEYS:
+            self.d[k].copy_(torch.from_numpy(np.ascontiguousarray(state[k])))
+
+    def save_state(self, path):
+        """state() written to an .npz file."""
+        np.savez(path, **self.state())
+
+    def load_state_file(self, path):
+        with np.load(path) as f:
+            self.load_state({k: f[k] for k in self.STATE_KEYS})
 
 
 def arrays_from_workload(w):
