@@ -4,7 +4,9 @@ an O(t) rs_match_index_build).
 
 ``python -m paper_2511_01282_gb300.retrieval_bench`` prints one JSON line per
 buffer length: device time of one query call (CUDA graph of 20 calls, CUDA
-events) for the scan and the index, and of one index build.  Buffers are
+events) for the scan and the index, and of one index build.  The calls run back
+to back, so buffers that fit in the L2 are read from it: the times compare the
+two methods rather than give the cold cost of a query.  Buffers are
 synthetic (seeded): V = 32000, segments of 8-64 tokens of which 30 % copy an
 earlier segment, scores uniform in [0, 1), key lengths 1-3.
 """
