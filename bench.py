@@ -285,6 +285,7 @@ def run_reference(args, rank, world):
             ests.append(est)
     est = statistics.median(ests)
     value = 1.0 / est
+    text += "; median of %d timed samples after %d untimed one(s)" % (args.steps, warm)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": est * 1e3, "higher_is_better": True,
