@@ -152,7 +152,10 @@ rs_status rs_entropy_gate_rows(const float *entropy, const int32_t *row_off,
  * R * ceil(V / 8192) <= RS_GATE_NOALLOC_MAX_PARTIALS (e.g. R <= 4096 rows at
  * V = 128256); larger calls return RS_ERR_CAPACITY without launching.
  * The first call on each device looks the array's device address up
- * (cudaGetSymbolAddress), so make that first call before any stream capture.
+ * (cudaGetSymbolAddress), so make that first call before any stream capture;
+ * the address is remembered per CUDA context, so the first call after a
+ * device reset (or from another context on the same device) looks it up
+ * again.
  * Nothing in the array needs to start at zero.  All calls share the array:
  * calls that overlap on the GPU (other streams, or unordered host threads)
  * race on it.  This call allocates nothing.

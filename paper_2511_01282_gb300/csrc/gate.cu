@@ -336,32 +336,64 @@ extern "C" rs_status rs_entropy_gate(const float *logits, int R, int V, const in
 }
 
 // ============================================================ no-allocation variant
-// rs_entropy_gate_noalloc runs the same two kernels as rs_entropy_gate, with
-// the per-chunk partials in the fixed device array below instead of a caller
-// workspace, for callers that cannot allocate device memory.  The array
-// (RS_GATE_NOALLOC_MAX_PARTIALS triples, 12 bytes each) lives on every GPU that
-// loads this library until the process exits.  It needs no initialisation:
-// every partial a call reads was written earlier by the same call.  All calls
-// share it, so calls that overlap on the GPU (different streams, or several
-// host threads without ordering) race on it.
+// rs_entropy_gate_noalloc runs the same three kernels as rs_entropy_gate
+// (entropy_partial, entropy_merge, gate_push), with the per-chunk partials in
+// the fixed device array below instead of a caller workspace, for callers
+// that cannot allocate device memory.  The array (RS_GATE_NOALLOC_MAX_PARTIALS
+// triples, 12 bytes each) lives on every GPU that loads this library until
+// the process exits.  It needs no initialisation: every partial a call reads
+// was written earlier by the same call.  All calls share it, so calls that
+// overlap on the GPU (different streams, or several host threads without
+// ordering) race on it.
 static __device__ __align__(256) Ent3 g_gate_scratch[RS_GATE_NOALLOC_MAX_PARTIALS];
 
-// Device address of g_gate_scratch on the current device, looked up once per
-// device (the host-side name is only a stand-in for the symbol).
+// Unique id of the calling thread's current CUDA context (0 when it cannot be
+// read).  Context ids are never reused within a process, so a device reset or
+// another context on the same device gives a new id.
+static unsigned long long current_context_id() {
+    typedef int (*ctx_get_current_t)(void **);
+    typedef int (*ctx_get_id_t)(void *, unsigned long long *);
+    static std::once_flag once;
+    static ctx_get_current_t get_current = nullptr;
+    static ctx_get_id_t get_id = nullptr;
+    std::call_once(once, [] {
+        void *a = nullptr, *b = nullptr;
+        cudaDriverEntryPointQueryResult qa, qb;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &a, 12000, cudaEnableDefault, &qa) ==
+                cudaSuccess && qa == cudaDriverEntryPointSuccess &&
+            cudaGetDriverEntryPointByVersion("cuCtxGetId", &b, 12000, cudaEnableDefault, &qb) == cudaSuccess &&
+            qb == cudaDriverEntryPointSuccess) {
+            get_current = reinterpret_cast<ctx_get_current_t>(a);
+            get_id = reinterpret_cast<ctx_get_id_t>(b);
+        }
+    });
+    if (!get_current || !get_id) return 0;
+    void *ctx = nullptr;
+    unsigned long long id = 0;
+    if (get_current(&ctx) != 0 || !ctx || get_id(ctx, &id) != 0) return 0;
+    return id;
+}
+
+// Device address of g_gate_scratch in the current context (the host-side name
+// is only a stand-in for the symbol).  Looked up with cudaGetSymbolAddress on
+// the first call in each context of each device and remembered with that
+// context's id; when the id cannot be read the address is looked up anew.
 static Ent3 *gate_scratch_address(int dev) {
     static std::mutex mu;
+    static unsigned long long ctx_of[64] = {0};
     static Ent3 *addr[64] = {nullptr};
     if (dev < 0 || dev >= 64) return nullptr;
     std::lock_guard<std::mutex> lk(mu);
-    if (!addr[dev]) {
-        void *ptr = nullptr;
-        cudaError_t e = cudaGetSymbolAddress(&ptr, g_gate_scratch);
-        if (e != cudaSuccess) {
-            set_error("rs_entropy_gate_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
-            return nullptr;
-        }
-        addr[dev] = static_cast<Ent3 *>(ptr);
+    const unsigned long long id = current_context_id();
+    if (id != 0 && ctx_of[dev] == id && addr[dev]) return addr[dev];
+    void *ptr = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&ptr, g_gate_scratch);
+    if (e != cudaSuccess) {
+        set_error("rs_entropy_gate_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+        return nullptr;
     }
+    addr[dev] = static_cast<Ent3 *>(ptr);
+    ctx_of[dev] = current_context_id();  // the lookup made the context current if it was not
     return addr[dev];
 }
 
