@@ -217,32 +217,47 @@ class VerifyStep:
         for k in self.STATE_KEYS:
             self.d[k].copy_(torch.from_numpy(self.host[k]))
 
-    def state(self):
+    def state(self, stream=None):
         """Checkpoint of the feedback state the decoding loop carries from step
         to step: the entropy history of the trigger (Section 3.2.1) and the EMA
-        score table of the selection (Eq. 4-5), as host arrays.  Synchronise
-        the stream the steps ran on first."""
+        score table of the selection (Eq. 4-5), as host arrays.  `stream` is
+        the stream the steps ran on (torch's current stream when None); it is
+        synchronised first, so the checkpoint follows every queued step."""
+        if self.d["hist"].is_cuda:
+            (stream if stream is not None else torch.cuda.current_stream()).synchronize()
         return {k: self.d[k].cpu().numpy().copy() for k in self.STATE_KEYS}
 
-    def load_state(self, state):
+    def load_state(self, state, stream=None):
         """Resume from a checkpoint taken by state() on a batch of the same
-        shapes (history [B, l], counts [B], scores parallel to the tokens)."""
+        shapes (history [B, l], counts [B], scores parallel to the tokens).
+
+        The copies are ordered on `stream` -- the stream the steps run on
+        (torch's current stream when None) -- behind any step still queued
+        there, which reads and writes the same buffers; the call returns once
+        the copies are done."""
         for k in self.STATE_KEYS:
             a = np.asarray(state[k])
             ref = self.host[k]
             if a.shape != ref.shape or a.dtype != ref.dtype:
                 raise ValueError("VerifyStep.load_state: %s is %s %s, this batch needs %s %s"
                                  % (k, a.dtype, a.shape, ref.dtype, ref.shape))
-        for k in self.STATE_KEYS:
-            self.d[k].copy_(torch.from_numpy(np.ascontiguousarray(state[k])))
+        if not self.d["hist"].is_cuda:
+            for k in self.STATE_KEYS:
+                self.d[k].copy_(torch.from_numpy(np.ascontiguousarray(state[k])))
+            return
+        st = stream if stream is not None else torch.cuda.current_stream()
+        with torch.cuda.stream(st):
+            for k in self.STATE_KEYS:
+                self.d[k].copy_(torch.from_numpy(np.ascontiguousarray(state[k])))
+        st.synchronize()
 
-    def save_state(self, path):
+    def save_state(self, path, stream=None):
         """state() written to an .npz file."""
-        np.savez(path, **self.state())
+        np.savez(path, **self.state(stream))
 
-    def load_state_file(self, path):
+    def load_state_file(self, path, stream=None):
         with np.load(path) as f:
-            self.load_state({k: f[k] for k in self.STATE_KEYS})
+            self.load_state({k: f[k] for k in self.STATE_KEYS}, stream)
 
 
 def arrays_from_workload(w):
