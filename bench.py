@@ -8,6 +8,7 @@ logits HBM bytes per step as GB/s and as a fraction of the measured peak.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the fp64 CPU oracle, timed on a sample
+  python bench.py --retrieval            # linear scan vs inverted index on long buffers
 
 Under torchrun each rank runs its own batch (requests are independent: weak
 scaling, no data-path collective); the timed region is bracketed by a barrier
@@ -53,6 +54,14 @@ def parse():
                     help="skip the end-to-end (host buffers) measurement: lean runs for profiling")
     ap.add_argument("--requests", type=int, default=0,
                     help="keep only the first N requests of the workload (small profiling cases)")
+    ap.add_argument("--soak-s", type=float, default=1.0,
+                    help="seconds of untimed step replays right before the timed steps, so that the "
+                         "sampled SM clocks cover the GPU under load")
+    ap.add_argument("--retrieval", action="store_true",
+                    help="instead of the step: rs_match_scan against the inverted index "
+                         "(rs_match_index_*) on long synthetic buffers, one JSON line per length")
+    ap.add_argument("--lengths", default="32768,262144,1048576,4194304",
+                    help="buffer lengths per request for --retrieval")
     return ap.parse_args()
 
 
@@ -230,15 +239,63 @@ def end_to_end(st, st2, graph, stream, K, W, barrier):
 
 
 # ------------------------------------------------------------------ CPU oracle sample
-def oracle_step_sample(w, budget_s, rows_cache={}):
-    """Time the oracle on a bounded sample of one step; return (est step s, sample text)."""
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def oracle_attn_rows(w, rows, workers):
+    """The oracle's attention on the given (node, head) rows, split into
+    disjoint row chunks run by `workers` host threads (the oracle's C code
+    releases the GIL; each row is computed on its own, so the split leaves its
+    arithmetic unchanged)."""
+    import concurrent.futures as cf
+
+    import numpy as np
+
+    import oracle
+    s = w.spec
+    rr = np.asarray(rows, dtype=np.int64).reshape(-1, 2)
+    if workers <= 1 or len(rr) < 2:
+        oracle.tree_attn(w.q, w.k, w.v, w.kv_off, w.ctx_len, w.node_off, w.parents, s.Hq, s.Hkv, s.D,
+                         s.D ** -0.5, rows=rr)
+        return
+    parts = np.array_split(rr, min(len(rr), workers * 4))
+    with cf.ThreadPoolExecutor(max_workers=workers) as ex:
+        list(ex.map(lambda part: oracle.tree_attn(w.q, w.k, w.v, w.kv_off, w.ctx_len, w.node_off, w.parents,
+                                                  s.Hq, s.Hkv, s.D, s.D ** -0.5, rows=part), parts))
+
+
+def oracle_entropy_rows(w, workers):
+    import concurrent.futures as cf
+
+    import numpy as np
+
+    import oracle
+    if workers <= 1:
+        return oracle.entropy_rows(w.logits)
+    parts = np.array_split(np.arange(w.R), min(w.R, workers))
+    with cf.ThreadPoolExecutor(max_workers=workers) as ex:
+        res = list(ex.map(lambda ix: oracle.entropy_rows(w.logits[ix[0]:ix[-1] + 1]) if len(ix) else
+                          np.zeros(0), parts))
+    return np.concatenate(res)
+
+
+def oracle_step_sample(w, budget_s, workers=1, rows_cache={}):
+    """Time the oracle on a bounded sample of one step on `workers` host
+    threads.  Entropy (rows split over the threads), gate, scan and accept run
+    over the whole batch; the attention runs on as many (node, head) rows of
+    request 0 as fit the budget and is scaled to all rows.  Returns (estimated
+    seconds per step, sample text, extrapolation record)."""
     import numpy as np
 
     import oracle
     s = w.spec
     f32 = lambda x: float(np.float32(x))  # noqa: E731
     t = time.perf_counter()
-    H = oracle.entropy_rows(w.logits)
+    H = oracle_entropy_rows(w, workers)
     oracle.gate(H, w.node_off, w.row_commit, w.hist, w.hist_n, s.l, f32(s.lambda_e), f32(s.theta_entropy))
     oracle.match_scan(w.tokens, w.tok_off, w.k_star_hint, w.scores, f32(s.theta_score), s.top_c, s.chain_len,
                       s.pos_cap)
@@ -247,25 +304,26 @@ def oracle_step_sample(w, budget_s, rows_cache={}):
     t_rest = time.perf_counter() - t
     # attention on (node, head) rows of request 0, as many as fit the budget
     n0, n1 = int(w.node_off[0]), int(w.node_off[1])
-    key = (id(w), budget_s)
+    total_rows = w.R * s.Hq
+    key = (id(w), budget_s, workers)
     if key not in rows_cache:
         t1 = time.perf_counter()
-        oracle.tree_attn(w.q, w.k, w.v, w.kv_off, w.ctx_len, w.node_off, w.parents, s.Hq, s.Hkv, s.D,
-                         s.D ** -0.5, rows=[(n0, 0)])
+        oracle_attn_rows(w, [(n0, 0)], 1)
         per_row = max(time.perf_counter() - t1, 1e-6)
-        rows_cache[key] = max(1, min(int(budget_s / per_row), (n1 - n0) * s.Hq))
+        rows_cache[key] = max(1, min(int(budget_s * workers / per_row), (n1 - n0) * s.Hq, total_rows))
     nrows = rows_cache[key]
     rows = [(n0 + (i % (n1 - n0)), (i // (n1 - n0)) % s.Hq) for i in range(nrows)]
     t = time.perf_counter()
-    oracle.tree_attn(w.q, w.k, w.v, w.kv_off, w.ctx_len, w.node_off, w.parents, s.Hq, s.Hkv, s.D, s.D ** -0.5,
-                     rows=rows)
+    oracle_attn_rows(w, rows, workers)
     t_attn = time.perf_counter() - t
-    frac = nrows / float(w.R * s.Hq)
-    est = t_rest + t_attn / frac
-    text = ("oracle on 1 host thread: entropy+gate+scan+accept over the whole batch (%.2f s) + attention "
-            "on %d of %d (node, head) rows (%.2f s), attention scaled by %.0fx"
-            % (t_rest, nrows, w.R * s.Hq, t_attn, 1 / frac))
-    return est, text
+    scale = total_rows / float(nrows)
+    est = t_rest + t_attn * scale
+    text = ("oracle on %d host thread(s): entropy+gate+scan+accept over the whole batch (%.2f s) + attention "
+            "on %d of %d (node, head) rows (%.2f s), attention scaled by %.1fx"
+            % (workers, t_rest, nrows, total_rows, t_attn, scale))
+    extra = {"rows_timed": nrows, "rows_total": total_rows, "scale": scale, "what": "attention rows",
+             "measured_s": t_rest + t_attn, "estimated_s": est}
+    return est, text, extra
 
 
 # ------------------------------------------------------------------ reference arm
@@ -274,24 +332,30 @@ def run_reference(args, rank, world):
         return 0
     import synth
     w = synth.make(args.workload, args.seed)
+    cores = host_cores()
     ests = []
-    text = ""
+    text, extra = "", {}
     warm = min(args.warmup, 1)
     # keep the whole run to a couple of minutes whatever K is
     budget = max(0.05, min(1.5, 90.0 / max(args.steps + warm, 1)))
+    t0 = time.perf_counter()
     for i in range(warm + args.steps):
-        est, text = oracle_step_sample(w, budget_s=budget)
+        est, text, extra = oracle_step_sample(w, budget_s=budget, workers=cores)
         if i >= warm:
             ests.append(est)
+    wall = time.perf_counter() - t0
     est = statistics.median(ests)
     value = 1.0 / est
     text += "; median of %d timed samples after %d untimed one(s)" % (args.steps, warm)
+    extra = dict(extra, samples=args.steps, wall_s=wall)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": est * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": WORKLOAD_TEXT[args.workload], "name": args.workload},
-        "cpu_baseline": {"value": value, "unit": "steps/s", "cores": 1, "kind": "oracle", "sample": text},
+        "extrapolated": extra,
+        "cpu_baseline": {"value": value, "unit": "steps/s", "cores": cores, "kind": "oracle", "sample": text,
+                         "extrapolated": extra},
         "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -300,7 +364,7 @@ def run_reference(args, rank, world):
 
 # ------------------------------------------------------------------ our arm
 def run_ours(args, rank, world, local_rank):
-    import numpy as np
+    import numpy as np  # noqa: F401
     import torch
 
     import __graft_entry__
@@ -339,53 +403,57 @@ def run_ours(args, rank, world, local_rank):
     with torch.cuda.graph(graph, stream=stream):
         st.step(stream)
 
-    def replay():
-        # a graph launches on the current stream: make that the timed stream
-        with torch.cuda.stream(stream):
-            graph.replay()
-
-    for _ in range(max(W, 3)):
-        replay()
-    torch.cuda.synchronize()
-
-    # L2: a step whose KV + logits fit in twice the L2 would run from the L2
-    # when replayed back to back; such steps (and calls) are timed one at a
-    # time, each after a write of twice the L2 size (outside the events)
+    # L2 flush before every timed step and call: a read of a buffer twice the
+    # L2 size evicts whatever the previous step or call left in the L2 and
+    # writes its dirty lines back, outside the timed region (a write-only
+    # flush would leave ~L2-size dirty lines for the timed work to write back)
     by = algorithmic_bytes(w)
     props = torch.cuda.get_device_properties(torch.cuda.current_device())
     l2 = int(getattr(props, "L2_cache_size", 0) or (126 << 20))
-    flush_buf = torch.empty(2 * l2, dtype=torch.uint8, device="cuda") if by["kv"] + by["logits"] < 2 * l2 else None
+    flush_buf = torch.ones(2 * l2 // 4, dtype=torch.int32, device="cuda")
+    flush_sink = torch.empty((), dtype=torch.int32, device="cuda")
+
+    def flush():
+        torch.amax(flush_buf, dim=0, out=flush_sink)
 
     def timed_replays(g, n):
-        """Device milliseconds of n replays of graph g on the timed stream."""
-        if flush_buf is None:
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            with torch.cuda.stream(stream):
-                a.record(stream)
-                for _ in range(n):
-                    g.replay()
-                b.record(stream)
-            torch.cuda.synchronize()
-            return a.elapsed_time(b)
+        """Device milliseconds of n replays of graph g on the timed stream,
+        each after an L2 flush that lies outside its pair of events."""
         ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
         with torch.cuda.stream(stream):
             for a, b in ev:
-                flush_buf.zero_()
+                flush()
                 a.record(stream)
                 g.replay()
                 b.record(stream)
         torch.cuda.synchronize()
         return sum(a.elapsed_time(b) for a, b in ev)
 
+    with torch.cuda.stream(stream):
+        for _ in range(max(W, 3)):
+            flush()
+            graph.replay()
+    torch.cuda.synchronize()
+
     clocks = ClockSampler(local_rank)
     clocks.start()
-    time.sleep(0.3)
 
     def barrier():
         if dist is not None:
             dist.barrier()
 
-    # ---- timed region: K graph replays
+    # ---- soak: untimed replays so the clock samples see the GPU under load
+    t_soak = time.perf_counter()
+    n_soak = 0
+    while time.perf_counter() - t_soak < args.soak_s:
+        with torch.cuda.stream(stream):
+            for _ in range(20):
+                flush()
+                graph.replay()
+        torch.cuda.synchronize()
+        n_soak += 20
+
+    # ---- timed region: K graph replays, each after an L2 flush
     barrier()
     torch.cuda.synchronize()
     local_ms = timed_replays(graph, K)
@@ -394,20 +462,18 @@ def run_ours(args, rank, world, local_rank):
     ms_per_step = t_ms / K
     value = job_rate(K, world, t_ms / 1e3)
 
-    # ---- per-call device time: a CUDA graph of n back-to-back calls, replayed
-    # on the timed stream between two events (no host launch gaps inside);
-    # with the L2 flush, a graph of one call timed n times
+    # ---- per-call device time: a CUDA graph of one call, replayed n times on
+    # the timed stream, each replay after an L2 flush (cold, as in the step)
     def time_call(fn, n):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
-            for _ in range(n if flush_buf is None else 1):
-                fn(stream)
+            fn(stream)
         with torch.cuda.stream(stream):
             g.replay()  # warm
         torch.cuda.synchronize()
-        return timed_replays(g, 1 if flush_buf is None else n) / n
+        return timed_replays(g, n) / n
 
-    n_call = max(5, min(K, 20))
+    n_call = max(10, min(K, 50))
     call_ms = {"gate_rows": time_call(st.gate_rows, n_call),
                "scan": time_call(lambda sm: st.scan(stream=sm), n_call),
                "attn": time_call(st.attn, n_call), "accept": time_call(lambda sm: st.accept(stream=sm), n_call),
@@ -431,44 +497,141 @@ def run_ours(args, rank, world, local_rank):
     clocks.stop()
 
     peaks, peak_kind = load_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+
+    def roof(name, nbytes, ms, what):
+        gbs = nbytes / (ms / 1e3) / 1e9
+        return {"kernel": name, "bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm,
+                "peak_kind": peak_kind, "algorithmic_bytes_per_launch": nbytes, "launch_ms": ms,
+                "timing": "cold: L2 flushed before each call; " + what}
+
     attn_s = call_ms["attn"] / 1e3
     achieved = by["attn"] / attn_s / 1e9
-    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
     step_gbs = (by["kv"] + by["logits"]) / (ms_per_step / 1e3) / 1e9
+    R, V = w.R, s.V
+    small_acc = R * (4 + 4 * s.beta + 4 + 4 + 4 + 4 + 1) + w.B * (4 * 4 + 64 * 4)
     line = {
         "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": K, "warmup": W,
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16+f32", "data": "synthetic",
         "config": {"workload": WORKLOAD_TEXT[args.workload] + (" (first %d requests)" % s.B if args.requests else ""),
                    "name": args.workload, "batch_per_gpu": s.B,
-                   "l2": ("no flush: every step streams %.2f GB of KV + logits, more than twice the %.0f MB L2"
-                          % ((by["kv"] + by["logits"]) / 1e9, l2 / 2**20) if flush_buf is None else
-                          "flushed: each timed step and call follows a %.0f MB write (twice the L2); "
-                          "the step's KV + logits (%.3f GB) would fit in L2" % (2 * l2 / 2**20,
-                                                                             (by["kv"] + by["logits"]) / 1e9)),
+                   "l2": ("flushed: each timed step and each timed call follows a read of a %.0f MB buffer "
+                          "(twice the L2), outside its events; the step moves %.3f GB of KV + logits"
+                          % (2 * l2 / 2**20, (by["kv"] + by["logits"]) / 1e9)),
                    "graph": "each step replays one CUDA graph of the 4 calls",
                    "step": "trigger on the row entropies rs_accept computed over the previous step's "
                            "verify logits (logits read once per step)"},
         "kv_logits_hbm": {"gbs": step_gbs, "frac": step_gbs / hbm, "peak": hbm, "peak_kind": peak_kind,
-                          "bytes_per_step": by["kv"] + by["logits"]},
+                          "bytes_per_step": by["kv"] + by["logits"],
+                          "note": "every byte comes from HBM: the L2 is flushed before each step"},
         "roofline": {"kernel": "rs_tree_verify_attn (prep + main + combine)", "bound": "hbm",
                      "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
                      "peak_kind": peak_kind, "algorithmic_bytes_per_launch": by["attn"],
                      "launch_ms": call_ms["attn"], "traffic": committed_traffic(args.workload),
-                     "tflops": by["flops"] / attn_s / 1e12},
+                     "tflops": by["flops"] / attn_s / 1e12,
+                     "tflops_frac_sustained": by["flops"] / attn_s / 1e12 / float(
+                         peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))},
+        "rooflines": {
+            "accept": roof("rs_accept (logits row pass + decisions)", R * V * 4 + small_acc, call_ms["accept"],
+                           "the whole call: row pass, and the decision kernel after it"),
+            "gate_from_logits": roof("rs_entropy_gate (logits row pass + history push)", R * V * 4,
+                                     call_ms["gate_from_logits"], "the whole call from the logits"),
+            "tree_sample": roof("rs_tree_sample (logits row pass + draws + walk)", R * V * 4,
+                                call_ms["tree_sample"], "the whole call"),
+        },
         "call_ms": call_ms,
         "e2e": ({"value": job_rate(K, world, e2e_s), "unit": "steps/s", "h2d_bytes_per_step": h2d,
                  "d2h_bytes_per_step": d2h} if K_e2e else None),
         "gpu_launches": launches_per_step * K,
         "launches_per_step": launches_per_step,
-        "clocks": clocks.summary(),
+        "clocks": dict(clocks.summary(), window="%.1f s soak of %d flushed step replays, then the timed steps, "
+                       "the per-call timings and the end-to-end loop" % (args.soak_s, n_soak)),
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        est, text = oracle_step_sample(w, budget_s=args.cpu_budget_s)
-        line["cpu_baseline"] = {"value": 1.0 / est, "unit": "steps/s", "cores": 1, "kind": "oracle",
-                                "sample": text}
+        cores = host_cores()
+        est, text, extra = oracle_step_sample(w, budget_s=args.cpu_budget_s, workers=cores)
+        est1, text1, extra1 = oracle_step_sample(w, budget_s=args.cpu_budget_s, workers=1)
+        line["cpu_baseline"] = {"value": 1.0 / est, "unit": "steps/s", "cores": cores, "kind": "oracle",
+                                "sample": text, "extrapolated": extra,
+                                "one_core": {"value": 1.0 / est1, "unit": "steps/s", "cores": 1, "sample": text1,
+                                             "extrapolated": extra1}}
     if rank == 0:
         print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------ retrieval leg
+def run_retrieval(args):
+    """rs_match_scan (O(t) per query) against rs_match_scan_indexed
+    (O(occurrences of the key's last token) per query, after an O(t)
+    rs_match_index_build) on long synthetic buffers: V = 32000, segments of
+    8-64 tokens of which 30 % copy an earlier segment, scores uniform in
+    [0, 1), key lengths 1-3.  Each call is timed cold (L2 flushed before each
+    of its replays); one JSON line per buffer length."""
+    import numpy as np
+    import torch
+
+    import __graft_entry__
+    from paper_2511_01282_gb300 import respec as rs
+    __graft_entry__.build()
+    V, B = 32000, 4
+    p = rs.params()
+    rng = np.random.default_rng(args.seed)
+    props = torch.cuda.get_device_properties(0)
+    l2 = int(getattr(props, "L2_cache_size", 0) or (126 << 20))
+    flush_buf = torch.ones(2 * l2 // 4, dtype=torch.int32, device="cuda")
+    sink = torch.empty((), dtype=torch.int32, device="cuda")
+    stream = torch.cuda.Stream()
+
+    def cold_us(fn, n=10):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(stream):
+            fn(stream)
+        torch.cuda.synchronize()
+        with torch.cuda.graph(g, stream=stream):
+            fn(stream)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+        with torch.cuda.stream(stream):
+            for a, b in ev:
+                torch.amax(flush_buf, dim=0, out=sink)
+                a.record(stream)
+                g.replay()
+                b.record(stream)
+        torch.cuda.synchronize()
+        return sum(a.elapsed_time(b) for a, b in ev) / n * 1e3
+
+    for t in [int(x) for x in args.lengths.split(",")]:
+        bufs = []
+        for _ in range(B):
+            out = []
+            while len(out) < t:
+                n = int(rng.integers(8, 65))
+                if out and rng.random() < 0.3:
+                    a = int(rng.integers(0, max(1, len(out) - n)))
+                    out += out[a:a + n]
+                else:
+                    out += rng.integers(0, V, n).tolist()
+            bufs.append(np.array(out[:t], np.int32))
+        tok_off = torch.tensor(np.concatenate([[0], np.cumsum([len(x) for x in bufs])]), dtype=torch.int64,
+                               device="cuda")
+        tokens = torch.from_numpy(np.concatenate(bufs)).cuda()
+        scores = torch.from_numpy(rng.random(tokens.numel()).astype(np.float32)).cuda()
+        ks = torch.tensor([1, 2, 3, 2][:B] * (B // 4 + 1), dtype=torch.int32, device="cuda")[:B].contiguous()
+        t_total = tokens.numel()
+        idx = torch.empty(rs.rs_match_index_bytes(B, V, t_total), dtype=torch.uint8, device="cuda")
+        z = lambda *sh: torch.zeros(sh, dtype=torch.int32, device="cuda")  # noqa: E731
+        o1 = [z(B), z(B, 1024), z(B, p.top_c), z(B, p.top_c), z(B, p.top_c, p.span_len), z(B), z(B)]
+        o2 = [z(B), z(B, 1024), z(B, p.top_c), z(B, p.top_c), z(B, p.top_c, p.span_len), z(B), z(B)]
+        scan_us = cold_us(lambda sm: rs.rs_match_scan(tokens, tok_off, B, ks, None, scores, p, 1024, *o1,
+                                                      stream=sm))
+        build_us = cold_us(lambda sm: rs.rs_match_index_build(tokens, tok_off, B, V, t_total, idx, stream=sm), n=3)
+        idx_us = cold_us(lambda sm: rs.rs_match_scan_indexed(tokens, tok_off, B, ks, None, scores, p, 1024,
+                                                             *o2, V, t_total, idx, stream=sm))
+        same = all(bool((a == b).all()) for a, b in zip(o1, o2))
+        print(json.dumps(dict(leg="retrieval", B=B, t=t, V=V, scan_us=round(scan_us, 2),
+                              indexed_us=round(idx_us, 2), build_us=round(build_us, 1), count=o1[0].tolist(),
+                              same_outputs=same, timing="cold: L2 flushed before each call")), flush=True)
     return 0
 
 
@@ -479,6 +642,8 @@ def main():
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         return run_reference(args, rank, world)
+    if args.retrieval:
+        return 0 if rank != 0 else run_retrieval(args)
     if world > 1:
         import torch
         import torch.distributed as dist
