@@ -160,6 +160,38 @@ def test_accept_chunk_counts(V, beta):
     check_accept(w, st)
 
 
+@pytest.mark.parametrize("V,B,beta,nodes", [(8, 3, 4, (1, 4)), (1024, 2, 5, (20, 40)), (4096, 2, 16, (20, 40)),
+                                               (4100, 3, 5, (20, 40)), (32000, 12, 5, (20, 40)),
+                                               (12288, 24, 16, (20, 40))])
+def test_logits_row_pass_sizes(V, B, beta, nodes):
+    # the gate and accept row passes on rows far shorter than one 8192-logit
+    # chunk, of exactly half and a little over half of one, and with more rows
+    # (B = 12, 24) than the GPU has SMs
+    w = synth.build(synth.small_spec(B=B, V=V, beta=beta, model_nodes=nodes), seed=V % 89 + B)
+    st = make_step(w)
+    check_gate(w, st)
+    check_accept(w, st)
+
+
+def test_logits_row_pass_masked_rows():
+    # rows with only a few finite logits (the rest -inf), fewer than beta in
+    # some: the top-beta list keeps -inf entries in id order, as the oracle
+    w = synth.build(synth.small_spec(B=3, V=6000, beta=8), seed=16)
+    rng = np.random.default_rng(16)
+    z = w.logits.copy()
+    for r in range(z.shape[0]):
+        keep = rng.choice(z.shape[1], size=int(rng.integers(1, 12)), replace=False)
+        mask = np.ones(z.shape[1], bool)
+        mask[keep] = False
+        if r % 3 == 0:  # also keep the row's draft children finite
+            mask[w.tree_tokens[w.node_off[0]:w.node_off[-1]]] = False
+        z[r, mask] = -np.inf
+    w.logits = z
+    st = make_step(w)
+    check_gate(w, st)
+    check_accept(w, st)
+
+
 def test_accept_without_entropy_output():
     w = synth.build(synth.small_spec(B=3, V=5000), seed=15)
     st = make_step(w)
