@@ -145,8 +145,11 @@ def greedy_reference(model, prompt, n_new):
 class SpecLoop:
     """One request decoded by the full step of Algorithm 1 (B = 1)."""
 
-    def __init__(self, target, draft, prompt, p, widths=(4, 3, 2), cap=4096, acc_cap=64):
+    def __init__(self, target, draft, prompt, p, widths=(4, 3, 2), cap=4096, acc_cap=64, trace=False):
         self.t, self.dr, self.p = target, draft, p
+        # with trace, every step appends host copies of each call's inputs and
+        # outputs to self.trace (for checking a run call by call)
+        self.trace = [] if trace else None
         self.widths = widths
         self.acc_cap = acc_cap
         dev = self.dev = target.device
@@ -206,8 +209,15 @@ class SpecLoop:
         i32 = lambda *s: torch.zeros(s, dtype=torch.int32, device=dev)  # noqa: E731
         sc = dict(count=i32(1), pos=i32(1, 16), sel_pos=i32(1, top_c), sel_len=i32(1, top_c),
                   spans=i32(1, top_c, L), n_sel=i32(1), status=i32(1))
+        tr = {} if self.trace is not None else None
+        host = lambda t: t.detach().cpu().numpy().copy()  # noqa: E731
+        if tr is not None:
+            tr["scan_in"] = dict(tokens=host(self.buf[:self.n]), k_star=host(self.k_star), gate_ok=host(self.ok),
+                                 scores=host(self.scores[:self.n]), pos_cap=16)
         rs.rs_match_scan(self.buf, tok_off, 1, self.k_star, self.ok, self.scores, p, 16, sc["count"], sc["pos"],
                          sc["sel_pos"], sc["sel_len"], sc["spans"], sc["n_sel"], sc["status"])
+        if tr is not None:
+            tr["scan_out"] = {k: host(v) for k, v in sc.items()}
         # 3. model drafts, then the chains under the root
         toks, par = self._draft_tree(root)
         source = [0] + [1] * (len(toks) - 1)
@@ -233,11 +243,18 @@ class SpecLoop:
                  acc_nodes=i32(1, self.acc_cap), bonus=i32(1), winner=i32(1),
                  commit=torch.zeros(N, dtype=torch.uint8, device=dev), status=i32(1))
         ws = torch.empty(max(rs.rs_accept_workspace_size(N, self.t.V, p.beta), 256), dtype=torch.uint8, device=dev)
+        if tr is not None:
+            tr["accept_in"] = dict(logits=host(logits), tokens=np.array(toks, np.int32), parents=np.array(par, np.int32),
+                                   source=np.array(source, np.uint8), chain=np.array(chain, np.int8),
+                                   sel_pos=host(sc["sel_pos"]), scores=host(self.scores[:self.n]),
+                                   acc_cap=self.acc_cap)
         rs.rs_accept(logits, N, self.t.V, node_off, 1, t_tok, t_par,
                      torch.tensor(source, dtype=torch.uint8, device=dev),
                      torch.tensor(chain, dtype=torch.int8, device=dev), sc["sel_pos"], tok_off, p, self.acc_cap,
                      o["argmax"], o["topk"], o["lse"], o["p_tok"], o["entropy"], o["acc_len"], o["acc_nodes"],
                      o["bonus"], o["winner"], o["commit"], self.scores, o["status"], ws)
+        if tr is not None:
+            tr["accept_out"] = dict({k: host(v) for k, v in o.items()}, scores=host(self.scores[:self.n]))
         # 5. commit: accepted tokens + bonus; K/V of the root and accepted slots into the prefix
         acc = o["acc_nodes"][0, :int(o["acc_len"][0])].cpu().numpy().tolist()
         argmax = o["argmax"].cpu().numpy()
@@ -250,8 +267,14 @@ class SpecLoop:
         self.dr.commit(self.dc, list(range(committed.numel())))
         self.n += len(new)
         # 1. (next step's) trigger from this verify's committed rows
+        if tr is not None:
+            tr["gate_in"] = dict(hist=host(self.hist), hist_n=host(self.hist_n))
         rs.rs_entropy_gate_rows(o["entropy"], node_off, o["commit"], 1, p, self.hist, self.hist_n,
                                 self.k_star, self.h_best, self.ok)
+        if tr is not None:
+            tr["gate_out"] = dict(hist=host(self.hist), hist_n=host(self.hist_n), k_star=host(self.k_star),
+                                  h_best=host(self.h_best), ok=host(self.ok))
+            self.trace.append(tr)
         st = self.stats
         st["steps"] += 1
         st["emitted"] += len(new)

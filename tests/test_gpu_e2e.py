@@ -12,11 +12,20 @@ its size; through the two layers and the head that is ~0.02 at logit std 6
 (measured: 0.011 at std 3), so 0.05 leaves margin while staying far below
 the median top-2 gap (~0.9).  Near-ties inside the margin may go either way; they
 are rare, and the test bounds how many.
+
+At the default tolerance (tau = 3, m = 2) the loop is replayed step by step
+through the oracle: every step's retrieval, acceptance (decisions, accepted
+path, bonus, winner, commit flags, updated scores) and trigger (history, k*,
+decision) must equal the oracle's on that step's recorded inputs, so the
+feedback state carried from step to step (Eq. 4-5 scores, the entropy
+history of Section 3.2.1) is pinned at every step.
 """
 import numpy as np
 import pytest
 import torch
 
+import oracle
+from gpu_helpers import ENT_TOL, LSE_REL, f32
 from paper_2511_01282_gb300 import respec as rs
 
 pytestmark = pytest.mark.gpu
@@ -79,3 +88,51 @@ def test_default_tolerance_loop_state():
     assert loop.tc["S"] == loop.n - 1 and loop.dc["S"] == loop.n - 1
     # on the model's own text the trigger fires and retrieved chains win steps
     assert s["triggered"] > 0 and s["retrieval_wins"] > 0
+
+
+def test_default_tolerance_loop_replayed_through_the_oracle():
+    from paper_2511_01282_gb300.e2e import SpecLoop, model_prompt
+    target, draft = _models(5)
+    prompt = model_prompt(target, 400, seed=5)
+    p = rs.params(span_len=8)
+    loop = SpecLoop(target, draft, prompt, p, trace=True)
+    loop.generate(160)
+    assert len(loop.trace) == loop.stats["steps"] > 20
+    seen = dict(trigger=0, chains=0, retrieval_win=0, relaxed=0)
+    for i, tr in enumerate(loop.trace):
+        si, so = tr["scan_in"], tr["scan_out"]
+        n = si["tokens"].size
+        tok_off = np.array([0, n], np.int64)
+        ms = oracle.match_scan(si["tokens"], tok_off, si["k_star"], si["scores"], f32(p.theta_score), p.top_c,
+                               p.span_len, si["pos_cap"], gate_ok=si["gate_ok"])
+        for k in ("count", "pos", "sel_pos", "sel_len", "spans", "n_sel", "status"):
+            assert (so[k] == ms[k]).all(), "step %d: scan %s" % (i, k)
+        ai, ao = tr["accept_in"], tr["accept_out"]
+        N = ai["tokens"].size
+        node_off = np.array([0, N], np.int32)
+        acc = oracle.accept(ai["logits"], node_off, ai["tokens"], ai["parents"], ai["source"], ai["chain"],
+                            ai["sel_pos"], tok_off, ai["scores"], p.beta, f32(p.tau), p.phi, p.m, f32(p.alpha),
+                            ai["acc_cap"])
+        for k in ("argmax", "topk", "acc_len", "acc_nodes", "bonus", "winner", "commit", "status", "scores"):
+            assert (ao[k] == acc[k]).all(), "step %d: accept %s" % (i, k)
+        assert np.allclose(ao["lse"], acc["lse"], rtol=LSE_REL, atol=1e-6), "step %d: lse" % i
+        H = oracle.entropy_rows(ai["logits"])
+        assert np.abs(ao["entropy"] - H).max() <= ENT_TOL, "step %d: entropy" % i
+        gi, go = tr["gate_in"], tr["gate_out"]
+        g = oracle.gate(ao["entropy"].astype(np.float64), node_off, ao["commit"], gi["hist"], gi["hist_n"], p.l,
+                        f32(p.lambda_e), f32(p.theta_entropy))
+        assert (go["k_star"] == g["k_star"]).all() and (go["ok"] == g["ok"]).all(), "step %d: trigger" % i
+        assert (go["h_best"] == g["h_best"].astype(np.float32)).all(), "step %d: h_best" % i
+        assert (go["hist"] == g["hist"].astype(np.float32)).all() and (go["hist_n"] == g["hist_n"]).all()
+        if i + 1 < len(loop.trace):  # the next step's scan is keyed and gated by this trigger
+            nxt = loop.trace[i + 1]["scan_in"]
+            assert (nxt["k_star"] == go["k_star"]).all() and (nxt["gate_ok"] == go["ok"]).all()
+            assert (nxt["scores"][:n] == ao["scores"]).all()  # the EMA state carries over
+        seen["trigger"] += int(go["ok"][0])
+        seen["chains"] += int(so["n_sel"][0] > 0)
+        seen["retrieval_win"] += int(ao["winner"][0] >= 0)
+        par = ai["parents"]
+        seen["relaxed"] += sum(int(ai["tokens"][a] != ao["argmax"][par[a]])
+                               for a in ao["acc_nodes"][0][:int(ao["acc_len"][0])])
+    # the replay covered the trigger firing, retrieved chains and retrieval wins
+    assert seen["trigger"] > 0 and seen["chains"] > 0 and seen["retrieval_win"] > 0, seen
