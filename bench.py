@@ -629,8 +629,28 @@ def run_retrieval(args):
         idx_us = cold_us(lambda sm: rs.rs_match_scan_indexed(tokens, tok_off, B, ks, None, scores, p, 1024,
                                                              *o2, V, t_total, idx, stream=sm))
         same = all(bool((a == b).all()) for a, b in zip(o1, o2))
+        # one decoding step's update: 8 committed tokens per request join the
+        # index (each timed replay appends the same 8 positions again: the
+        # index is rebuilt on the shorter buffers before every replay)
+        grown = [np.concatenate([x, x[-8:]]) for x in bufs]
+        g_off = torch.tensor(np.concatenate([[0], np.cumsum([len(x) for x in grown])]), dtype=torch.int64,
+                             device="cuda")
+        g_tok = torch.from_numpy(np.concatenate(grown)).cuda()
+        st_app = torch.zeros(B, dtype=torch.int32, device="cuda")
+        app_us = []
+        for _ in range(5):  # eager: the flush keeps the GPU busy while the append is enqueued
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            with torch.cuda.stream(stream):
+                rs.rs_match_index_build(tokens, tok_off, B, V, t_total, idx, stream=stream)
+                torch.amax(flush_buf, dim=0, out=sink)
+                a.record(stream)
+                rs.rs_match_index_append(g_tok, g_off, B, V, t_total, idx, st_app, stream=stream)
+                b.record(stream)
+            torch.cuda.synchronize()
+            app_us.append(a.elapsed_time(b) * 1e3)
         print(json.dumps(dict(leg="retrieval", B=B, t=t, V=V, scan_us=round(scan_us, 2),
-                              indexed_us=round(idx_us, 2), build_us=round(build_us, 1), count=o1[0].tolist(),
+                              indexed_us=round(idx_us, 2), build_us=round(build_us, 1),
+                              append8_us=round(sorted(app_us)[2], 2), count=o1[0].tolist(),
                               same_outputs=same, timing="cold: L2 flushed before each call")), flush=True)
     return 0
 

@@ -293,30 +293,45 @@ rs_status rs_accept(const float *logits, int R, int V, const int32_t *node_off, 
                     int32_t *status, void *workspace, size_t workspace_bytes, void *stream);
 
 /* ============================================ rs_match_index (NEXT-4) ====
- * An index for Section 3.3's retrieval on long buffers.  Algorithm 1 asks
- * its suffix automaton two things about the key (the buffer's last
- * k <= RS_MAX_L tokens): Contains and RetrievePositions.  Both are answered
- * exactly from an inverted index: for every token id, the ascending list of
- * positions holding it; the positions holding the key's last token are the
- * candidates, verified against the key's other tokens.  A query costs
- * O(occurrences of that token) instead of rs_match_scan's O(t).
+ * An index for Section 3.3's retrieval on long buffers, kept current step by
+ * step.  Algorithm 1 asks its suffix automaton two things about the key (the
+ * buffer's last k <= RS_MAX_L tokens), Contains and RetrievePositions, and
+ * after each step adds the committed tokens to it (Update).  Both questions
+ * are answered exactly from an inverted index: for every token id, the
+ * ascending list of positions holding it; the positions holding the key's
+ * last token are the candidates, verified against the key's other tokens.  A
+ * query costs O(occurrences of that token) instead of rs_match_scan's O(t);
+ * an update costs O(tokens added).
  *
  * rs_match_index_bytes(B, V, t_total): device bytes of an index over B
- *   buffers of ids in [0, V) (others share one bucket) with t_total tokens
- *   in all (tok_off[B] at build time).
+ *   buffers of ids in [0, V) (others share one bucket) holding t_total tokens
+ *   in all at build time (tok_off[B] then), including the build's scratch.
+ *   Each id's list has room for a quarter more positions than it held at
+ *   build time (plus two), and each request has an overflow list of 4096
+ *   positions for ids whose room is used up.
  * rs_match_index_build: indexes tokens[tok_off[b] .. tok_off[b+1]) of every
  *   request (the index remembers each request's length and offset).  The
- *   caller owns `index`; nothing in it needs initialising.
+ *   caller owns `index`; nothing in it needs initialising.  Requires
+ *   ceil(log2(V + 1)) + ceil(log2(B)) <= 32 (RS_ERR_UNSUPPORTED otherwise).
+ * rs_match_index_append: adds the tokens appended to each request's buffer
+ *   since the build or the last append: positions built .. t_b - 1, where t_b
+ *   = tok_off[b+1] - tok_off[b] now (positions are relative to the request's
+ *   first token, so the buffers may be laid out anew between calls; the
+ *   tokens already indexed must not change).  V and t_total as given to the
+ *   build.  status [B] int32 (or NULL): RS_ST_TRUNCATED when some positions
+ *   could not be indexed (an id's room and the overflow list both full): they
+ *   and every later position are then tested one by one by the queries until
+ *   the next build.  One CTA per request.
  * rs_match_scan_indexed: rs_match_scan's inputs, outputs and meaning, plus
- *   V, t_total (as given to the build) and the index.  tok_off may have grown
- *   since the build (tokens appended at the end of a request's buffer, its
- *   first token's offset unchanged relative to its own buffer): positions
- *   at or after the length indexed are tested one by one, so rebuild when
- *   that tail gets long.  One CTA per request.
+ *   V, t_total (as given to the build) and the index.  Positions the index
+ *   does not hold (appended without rs_match_index_append, or left out as
+ *   above) are tested one by one.  One CTA per request.
  */
 size_t rs_match_index_bytes(int B, int V, int64_t t_total);
 rs_status rs_match_index_build(const int32_t *tokens, const int64_t *tok_off, int B, int V, int64_t t_total,
                                void *index, size_t index_bytes, void *stream);
+rs_status rs_match_index_append(const int32_t *tokens, const int64_t *tok_off, int B, int V, int64_t t_total,
+                                void *index, size_t index_bytes, int32_t *status, void *stream);
 rs_status rs_match_scan_indexed(const int32_t *tokens, const int64_t *tok_off, int B, const int32_t *k_star,
                                 const uint8_t *gate_ok, const float *scores, rs_params p, int pos_cap,
                                 int32_t *count, int32_t *pos, int32_t *sel_pos, int32_t *sel_len,

@@ -67,6 +67,7 @@ _SIGS = {
                             _P]),
     "rs_match_index_bytes": (C.c_size_t, [C.c_int, C.c_int, C.c_int64]),
     "rs_match_index_build": (C.c_int, [_P, _P, C.c_int, C.c_int, C.c_int64, _P, C.c_size_t, _P]),
+    "rs_match_index_append": (C.c_int, [_P, _P, C.c_int, C.c_int, C.c_int64, _P, C.c_size_t, _P, _P]),
     "rs_match_scan_indexed": (C.c_int, [_P, _P, C.c_int, _P, _P, _P, rs_params, C.c_int] + [_P] * 7
                               + [C.c_int, C.c_int64, _P, C.c_size_t, _P]),
     "rs_tree_sample_workspace_size": (C.c_size_t, [C.c_int, C.c_int]),
@@ -201,6 +202,11 @@ def rs_match_index_bytes(B, V, t_total):
 def rs_match_index_build(tokens, tok_off, B, V, t_total, index, stream=None):
     _check(lib().rs_match_index_build(_ptr(tokens), _ptr(tok_off), B, V, t_total, _ptr(index),
                                       index.numel() * index.element_size(), _stream(stream)))
+
+
+def rs_match_index_append(tokens, tok_off, B, V, t_total, index, status=None, stream=None):
+    _check(lib().rs_match_index_append(_ptr(tokens), _ptr(tok_off), B, V, t_total, _ptr(index),
+                                       index.numel() * index.element_size(), _ptr(status), _stream(stream)))
 
 
 def rs_match_scan_indexed(tokens, tok_off, B, k_star, gate_ok, scores, p, pos_cap, count, pos, sel_pos,

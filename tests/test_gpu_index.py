@@ -121,3 +121,70 @@ def test_skips_and_truncation():
     for key in ("count", "pos", "sel_pos", "sel_len", "spans", "n_sel"):
         assert (got[key] == ref[key]).all(), key
     assert got["status"][0] & rs.RS_ST_TRUNCATED
+
+
+def _grow(rng, buf, n, V, copy_prob):
+    """Append n tokens to buf: copies of earlier spans (so keys recur) or fresh ids."""
+    out = list(buf)
+    while len(out) < len(buf) + n:
+        if len(out) > 8 and rng.random() < copy_prob:
+            a = int(rng.integers(0, len(out) - 4))
+            out += out[a:a + int(rng.integers(2, 6))]
+        else:
+            out.append(int(rng.integers(0, V)))
+    return np.array(out[:len(buf) + n], np.int32)
+
+
+def _layout(bufs):
+    tok_off = np.concatenate([[0], np.cumsum([len(x) for x in bufs])]).astype(np.int64)
+    return np.concatenate(bufs).astype(np.int32), tok_off
+
+
+def test_append_matches_the_oracle_after_every_step():
+    # Algorithm 1's update: each step appends a few committed tokens to every
+    # request's buffer and rs_match_index_append adds them to the index; after
+    # every step the indexed retrieval equals the oracle's scan bit for bit
+    rng = np.random.default_rng(41)
+    V = 500
+    bufs = [_grow(rng, np.zeros(0, np.int32), n, V, 0.5) for n in (2000, 50, 5000, 1)]
+    tokens, tok_off = _layout(bufs)
+    idx, t_total = build_index(tokens, tok_off, V)
+    status = torch.full((4,), -1, dtype=torch.int32, device="cuda")
+    for step in range(40):
+        bufs = [_grow(rng, b, int(rng.integers(0, 13)), V, 0.6) for b in bufs]
+        tokens, tok_off = _layout(bufs)
+        rs.rs_match_index_append(_cuda(tokens), _cuda(tok_off), 4, V, t_total, idx, status)
+        torch.cuda.synchronize()
+        assert (status.cpu().numpy() == 0).all()
+        scores = rng.random(len(tokens)).astype(np.float32)
+        ks = rng.integers(1, 4, 4).astype(np.int32)
+        got = compare(tokens, tok_off, ks, None, scores, 0.25, 3, 8, 64, V, idx=idx, t_total=t_total)
+    assert (got["count"] > 0).any()
+
+
+def test_append_overflow_then_linear_tail():
+    # one id appended far beyond its room: the overflow list takes 4096
+    # positions, then indexing stops (RS_ST_TRUNCATED) and the later positions
+    # are tested one by one; the answers stay exact throughout and after a
+    # rebuild
+    rng = np.random.default_rng(43)
+    V = 20
+    bufs = [rng.integers(0, V, 100).astype(np.int32) for _ in range(2)]
+    tokens, tok_off = _layout(bufs)
+    idx, t_total = build_index(tokens, tok_off, V)
+    status = torch.full((2,), -1, dtype=torch.int32, device="cuda")
+    seen = []
+    for n in (3000, 2000, 7):
+        bufs = [np.concatenate([bufs[0], np.full(n, 7, np.int32)]), _grow(rng, bufs[1], 5, V, 0.5)]
+        tokens, tok_off = _layout(bufs)
+        rs.rs_match_index_append(_cuda(tokens), _cuda(tok_off), 2, V, t_total, idx, status)
+        torch.cuda.synchronize()
+        seen.append(status.cpu().numpy().copy())
+        scores = rng.random(len(tokens)).astype(np.float32)
+        for k in (1, 2, 3):
+            compare(tokens, tok_off, np.array([k, k], np.int32), None, scores, 0.3, 3, 8, 300, V, idx=idx,
+                    t_total=t_total)
+    assert seen[0][0] == 0 and seen[1][0] == rs.RS_ST_TRUNCATED and seen[2][0] == rs.RS_ST_TRUNCATED
+    assert (np.array(seen)[:, 1] == 0).all()
+    # a fresh build holds everything again
+    compare(tokens, tok_off, np.array([2, 3], np.int32), None, scores, 0.3, 3, 8, 300, V)
