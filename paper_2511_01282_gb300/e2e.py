@@ -11,7 +11,9 @@ plain torch matmuls.  Every step:
 
   1. trigger: ``rs_entropy_gate_rows`` on the previous verify's row entropies
      (k*, entropy_ok; nothing fires until the history has entries);
-  2. retrieval: ``rs_match_scan`` over the committed tokens -> up to top_c
+  2. retrieval: ``rs_match_scan`` over the committed tokens (or, with
+     ``retrieval="index"``, ``rs_match_scan_indexed`` on an index that
+     ``rs_match_index_append`` brings up to date) -> up to top_c
      continuations, attached under the root as retrieved chains;
   3. model drafts: the draft model expands a top-w tree level by level;
   4. verification: one target forward over the whole tree, then
@@ -145,8 +147,14 @@ def greedy_reference(model, prompt, n_new):
 class SpecLoop:
     """One request decoded by the full step of Algorithm 1 (B = 1)."""
 
-    def __init__(self, target, draft, prompt, p, widths=(4, 3, 2), cap=4096, acc_cap=64, trace=False):
+    def __init__(self, target, draft, prompt, p, widths=(4, 3, 2), cap=4096, acc_cap=64, trace=False,
+                 retrieval="scan"):
         self.t, self.dr, self.p = target, draft, p
+        # retrieval: "scan" (rs_match_scan over the buffer) or "index" (an
+        # index built over the prompt, the committed tokens appended to it
+        # every step, queried with rs_match_scan_indexed)
+        assert retrieval in ("scan", "index")
+        self.retrieval = retrieval
         # with trace, every step appends host copies of each call's inputs and
         # outputs to self.trace (for checking a run call by call)
         self.trace = [] if trace else None
@@ -177,6 +185,12 @@ class SpecLoop:
                 m.forward_tree(cache, toks, self._chain_parents(toks.numel()), self.ws_attn)
                 m.commit(cache, list(range(toks.numel())))
         self.stats = dict(steps=0, emitted=0, triggered=0, retrieval_wins=0, model_wins=0, relaxed=0)
+        if retrieval == "index":
+            self.idx_t = len(prompt)
+            self.idx = torch.empty(rs.rs_match_index_bytes(1, target.V, self.idx_t), dtype=torch.uint8, device=dev)
+            self.idx_status = torch.zeros(1, dtype=torch.int32, device=dev)
+            rs.rs_match_index_build(self.buf, torch.tensor([0, self.n], dtype=torch.int64, device=dev), 1, target.V,
+                                    self.idx_t, self.idx)
 
     def _chain_parents(self, n):
         return torch.arange(-1, n - 1, dtype=torch.int32, device=self.dev)
@@ -214,8 +228,15 @@ class SpecLoop:
         if tr is not None:
             tr["scan_in"] = dict(tokens=host(self.buf[:self.n]), k_star=host(self.k_star), gate_ok=host(self.ok),
                                  scores=host(self.scores[:self.n]), pos_cap=16)
-        rs.rs_match_scan(self.buf, tok_off, 1, self.k_star, self.ok, self.scores, p, 16, sc["count"], sc["pos"],
-                         sc["sel_pos"], sc["sel_len"], sc["spans"], sc["n_sel"], sc["status"])
+        if self.retrieval == "index":
+            # the previous step's committed tokens join the index (Algorithm 1's update), then the query
+            rs.rs_match_index_append(self.buf, tok_off, 1, self.t.V, self.idx_t, self.idx, self.idx_status)
+            rs.rs_match_scan_indexed(self.buf, tok_off, 1, self.k_star, self.ok, self.scores, p, 16, sc["count"],
+                                     sc["pos"], sc["sel_pos"], sc["sel_len"], sc["spans"], sc["n_sel"], sc["status"],
+                                     self.t.V, self.idx_t, self.idx)
+        else:
+            rs.rs_match_scan(self.buf, tok_off, 1, self.k_star, self.ok, self.scores, p, 16, sc["count"], sc["pos"],
+                             sc["sel_pos"], sc["sel_len"], sc["spans"], sc["n_sel"], sc["status"])
         if tr is not None:
             tr["scan_out"] = {k: host(v) for k, v in sc.items()}
         # 3. model drafts, then the chains under the root

@@ -90,12 +90,16 @@ def test_default_tolerance_loop_state():
     assert s["triggered"] > 0 and s["retrieval_wins"] > 0
 
 
-def test_default_tolerance_loop_replayed_through_the_oracle():
+@pytest.mark.parametrize("retrieval", ["scan", "index"])
+def test_default_tolerance_loop_replayed_through_the_oracle(retrieval):
+    # retrieval="index": the index is built over the prompt and every step's
+    # committed tokens are appended to it before the query, so the replay also
+    # pins the indexed retrieval, step after step, inside a live loop
     from paper_2511_01282_gb300.e2e import SpecLoop, model_prompt
     target, draft = _models(5)
     prompt = model_prompt(target, 400, seed=5)
     p = rs.params(span_len=8)
-    loop = SpecLoop(target, draft, prompt, p, trace=True)
+    loop = SpecLoop(target, draft, prompt, p, trace=True, retrieval=retrieval)
     loop.generate(160)
     assert len(loop.trace) == loop.stats["steps"] > 20
     seen = dict(trigger=0, chains=0, retrieval_win=0, relaxed=0)
@@ -136,3 +140,5 @@ def test_default_tolerance_loop_replayed_through_the_oracle():
                                for a in ao["acc_nodes"][0][:int(ao["acc_len"][0])])
     # the replay covered the trigger firing, retrieved chains and retrieval wins
     assert seen["trigger"] > 0 and seen["chains"] > 0 and seen["retrieval_win"] > 0, seen
+    if retrieval == "index":
+        assert int(loop.idx_status[0]) == 0  # every committed token went into the index
