@@ -374,12 +374,14 @@ accept_merge(const VI *__restrict__ cand, const MS *__restrict__ part, int nchun
 }
 
 constexpr int kDecThreads = 512;
+static_assert(kDecThreads >= RS_MAX_NODES + RS_MAX_TOPC, "one thread per node plus one per selection");
 constexpr int kNodeWords = RS_MAX_NODES / 32;
 
 // One CTA per request.  Every global read happens in two dependent rounds
-// at the start (the tree, the row statistics and the selected positions'
-// scores; then the logit of each node's token in its parent's row); the rest
-// works on shared memory.  Per node it precomputes the greedy match
+// at the start (the tree and the row statistics, then the logit of each
+// node's token in its parent's row; the selected positions and their scores
+// are read by other threads at the same time); the rest works on shared
+// memory.  Per node it precomputes the greedy match
 // (token == argmax of the parent row) and the relaxed check of Eq. 6-7
 // (token among the parent row's top beta and max logit - token logit <= tau
 // in fp64), so each chain's look-ahead walk and each model node's path check
@@ -431,43 +433,62 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
     }
     const long long t0 = tok_off[b];
     const long long t = tok_off[b + 1] - t0;
-    if (tid < top_c) {  // the selected positions and their scores (Eq. 4-5 inputs)
-        const int pos = sel_pos[(long long)b * top_c + tid];
-        s_selp[tid] = pos;
-        s_selS[tid] = (pos >= 0 && (long long)pos < t) ? scores[t0 + pos] : 0.f;
-    }
-    __syncthreads();
 
-    // ---- the two dependent read rounds: tree and row statistics, then token logits ----
-    if (st == 0) {
-        for (int i = tid; i < N; i += kDecThreads) {
-            const int pa = parents[n0 + i];
-            const int sr = source[n0 + i];
-            const int ch = chain[n0 + i];
-            const int tk = tokens[n0 + i];
-            s_arg[i] = argmax[n0 + i];
-            s_zmax[i] = rowmax[n0 + i];
-            s_par[i] = pa;
-            s_tok[i] = tk;
-            s_src[i] = (uint8_t)sr;
-            s_chn[i] = (int8_t)ch;
-            commit[n0 + i] = 0;
-            bool bad;
-            if (i == 0) bad = (pa != -1 || sr != 0 || ch != -1);
-            else bad = (pa < 0 || pa >= i || sr < 1 || sr > 2 || (sr == 2 && (ch < 0 || ch >= top_c)) ||
-                        (sr == 1 && ch != -1) || tk < 0 || tk >= V);
-            if (bad) {
-                atomicOr(&s_bad, 1);
-            } else if (i == 0) {
-                p_tok[n0] = 1.f;
-            } else {
-                const float z = logits[(long long)(n0 + pa) * V + tk];
-                s_ztok[i] = z;
-                p_tok[n0 + i] = __expf(z - lse[n0 + pa]);
-            }
+    // ---- every global read up front.  Node = tid (N <= RS_MAX_NODES, one
+    // per thread): its tree entries and row statistics, then its token's
+    // logit in the parent's row (two dependent rounds); meanwhile threads
+    // RS_MAX_NODES .. read the selected positions and their scores (Eq. 4-5
+    // inputs) and every thread reads top-beta ids ----
+    const int node = tid;
+    int r_pa = 0, r_sr = 0, r_ch = 0, r_tk = 0, r_am = 0;
+    float r_zmax = 0.f, r_z = 0.f, r_lp = 0.f;
+    bool r_bad = false;
+    if (st == 0 && node < N) {
+        r_pa = parents[n0 + node];
+        r_sr = source[n0 + node];
+        r_ch = chain[n0 + node];
+        r_tk = tokens[n0 + node];
+        r_am = argmax[n0 + node];
+        r_zmax = rowmax[n0 + node];
+        if (node == 0) r_bad = (r_pa != -1 || r_sr != 0 || r_ch != -1);
+        else r_bad = (r_pa < 0 || r_pa >= node || r_sr < 1 || r_sr > 2 || (r_sr == 2 && (r_ch < 0 || r_ch >= top_c)) ||
+                    (r_sr == 1 && r_ch != -1) || r_tk < 0 || r_tk >= V);
+        if (!r_bad && node > 0) {
+            r_z = logits[(long long)(n0 + r_pa) * V + r_tk];
+            r_lp = lse[n0 + r_pa];
         }
+    }
+    const int js = tid - RS_MAX_NODES;
+    int selp = -1;
+    float selS = 0.f;
+    if (js >= 0 && js < top_c) {
+        selp = sel_pos[(long long)b * top_c + js];
+        selS = (selp >= 0 && (long long)selp < t) ? scores[t0 + selp] : 0.f;
+    }
+    if (st == 0)
         for (int x = tid; x < N * beta; x += kDecThreads)
             s_top[(x / beta) * RS_MAX_BETA + (x % beta)] = topk[(long long)n0 * beta + x];
+    __syncthreads();  // s_bad, s_best and s_stt are initialised
+    if (js >= 0 && js < top_c) {
+        s_selp[js] = selp;
+        s_selS[js] = selS;
+    }
+    if (st == 0 && node < N) {
+        s_arg[node] = r_am;
+        s_zmax[node] = r_zmax;
+        s_par[node] = r_pa;
+        s_tok[node] = r_tk;
+        s_src[node] = (uint8_t)r_sr;
+        s_chn[node] = (int8_t)r_ch;
+        commit[n0 + node] = 0;
+        if (r_bad) {
+            atomicOr(&s_bad, 1);
+        } else if (node == 0) {
+            p_tok[n0] = 1.f;
+        } else {
+            s_ztok[node] = r_z;
+            p_tok[n0 + node] = __expf(r_z - r_lp);
+        }
     }
     __syncthreads();
     const bool ok1 = st == 0 && s_bad == 0;
