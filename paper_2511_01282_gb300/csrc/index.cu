@@ -151,7 +151,9 @@ index_count(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_
 }
 
 // (3) per request: bucket starts (prefix of the rooms) and the sorted starts
-// (prefix of the counts); len keeps the counts
+// (prefix of the counts); len keeps the counts.  Each thread takes kOffPer
+// consecutive buckets, so one round of the block covers 8192 of them.
+constexpr int kOffPer = 8;
 __global__ void __launch_bounds__(kIdxThreads)
 index_offsets(int V, IndexView ix) {
     pdl_enter();
@@ -163,11 +165,17 @@ index_offsets(int V, IndexView ix) {
     int32_t *sstart = ix.sstart + (long long)b * (V + 1);
     if (threadIdx.x < 2) s_carry[threadIdx.x] = 0;
     __syncthreads();
-    for (int base = 0; base < V + 1; base += kIdxThreads) {
-        const int i = base + threadIdx.x;
-        const int c = i < V + 1 ? cnt[i] : 0;
-        int x0 = i < V + 1 ? room_of(c) : 0, x1 = c;
-        const int v0 = x0, v1 = x1;
+    for (int base = 0; base < V + 1; base += kIdxThreads * kOffPer) {
+        const int i0 = base + threadIdx.x * kOffPer;
+        int c[kOffPer];
+        int r0 = 0, r1 = 0;  // this thread's rooms and counts
+#pragma unroll
+        for (int q = 0; q < kOffPer; ++q) {
+            c[q] = i0 + q < V + 1 ? cnt[i0 + q] : 0;
+            r0 += i0 + q < V + 1 ? room_of(c[q]) : 0;
+            r1 += c[q];
+        }
+        int x0 = r0, x1 = r1;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int y0 = __shfl_up_sync(0xffffffffu, x0, o), y1 = __shfl_up_sync(0xffffffffu, x1, o);
@@ -188,9 +196,15 @@ index_offsets(int V, IndexView ix) {
             t0s += s_w[0][w];
             t1s += s_w[1][w];
         }
-        if (i < V + 1) {
-            start[i] = s_carry[0] + b0 + x0 - v0;
-            sstart[i] = s_carry[1] + b1 + x1 - v1;
+        int e0 = s_carry[0] + b0 + x0 - r0, e1 = s_carry[1] + b1 + x1 - r1;
+#pragma unroll
+        for (int q = 0; q < kOffPer; ++q) {
+            if (i0 + q < V + 1) {
+                start[i0 + q] = e0;
+                sstart[i0 + q] = e1;
+                e0 += room_of(c[q]);
+                e1 += c[q];
+            }
         }
         __syncthreads();
         if (threadIdx.x == 0) {
