@@ -68,6 +68,13 @@ typedef enum {
                                wait, ~2 s; the environment variable
                                RS_DEBUG_WAIT_LIMIT, in clock cycles, shortens it
                                for tests); the request's outputs are invalid   */
+#define RS_ST_BAD_OFFSET 32 /* the request's range in an offsets array lies
+                               outside the arrays it indexes (a negative start
+                               or length, or an end past R, kv_rows, t_total or
+                               the array's last entry): the kernels check every
+                               range they read from device memory before they
+                               index with it, skip the request and leave every
+                               array outside their own outputs untouched     */
 
 /* -------------------------------------------------------------- parameters */
 /* Hyper-parameters of Algorithm 1 (its inputs), Eq. 6-7 and Section 3.4.
@@ -96,6 +103,15 @@ const char *rs_version(void);
 
 /* Number of kernels this library has launched in this process. */
 uint64_t rs_launch_count(void);
+
+/* Offsets arrays hold device data the host cannot check, so each kernel
+ * checks the ranges it reads (see RS_ST_BAD_OFFSET): node_off / row_off
+ * against R (or their last entry), tok_off against its last entry (the token
+ * and score buffers hold tok_off[B] entries) or the index's t_total, kv_off +
+ * ctx_len + node count against kv_rows.  rs_entropy_gate and
+ * rs_entropy_gate_rows have no status output: a request whose row range is
+ * out of bounds pushes no entropies (its trigger is evaluated on its history
+ * as it was). */
 
 /* ===================================================== rs_entropy_gate ====
  * Section 3.2.1 (Eq. 1: mean predictive entropy of a key; Eq. 2: C_k =

@@ -388,7 +388,7 @@ constexpr int kNodeWords = RS_MAX_NODES / 32;
 // read only flags.  Chain c's nodes are ranked by popcounts of per-chain
 // membership masks (one warp ballot per 32 nodes).
 __global__ void __launch_bounds__(kDecThreads)
-accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict__ node_off,
+accept_decide(const float *__restrict__ logits, int R, int V, const int32_t *__restrict__ node_off,
               const int32_t *__restrict__ tokens, const int32_t *__restrict__ parents,
               const uint8_t *__restrict__ source, const int8_t *__restrict__ chain,
               const int32_t *__restrict__ sel_pos, const int64_t *__restrict__ tok_off, rs_params p,
@@ -423,16 +423,21 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
     __shared__ int s_bad, s_stt, s_win, s_dup;
     __shared__ int s_best;  // (depth << 16) | (0xffff - node)
 
+    // the request's rows must lie in [0, R) and its buffer in the score table
+    // (tok_off[B] entries); outside them nothing is read or written
+    const bool rows_ok = n0 >= 0 && N >= 0 && (long long)n0 + N <= R;
+    const long long t0 = tok_off[b];
+    const long long t = tok_off[b + 1] - t0;
+    const bool tok_ok = t0 >= 0 && t >= 0 && t0 + t <= tok_off[gridDim.x];
     int st = 0;
-    if (N > RS_MAX_NODES) st = RS_ST_TOO_LARGE;
+    if (!rows_ok || !tok_ok) st = RS_ST_BAD_OFFSET;
+    else if (N > RS_MAX_NODES) st = RS_ST_TOO_LARGE;
     else if (N < 1) st = RS_ST_BAD_TREE;
     if (tid == 0) {
         s_bad = 0;
         s_best = 0;
         s_stt = 0;
     }
-    const long long t0 = tok_off[b];
-    const long long t = tok_off[b + 1] - t0;
 
     // ---- every global read up front.  Node = tid (N <= RS_MAX_NODES, one
     // per thread): its tree entries and row statistics, then its token's
@@ -463,7 +468,7 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
     float selS = 0.f;
     if (js >= 0 && js < top_c) {
         selp = sel_pos[(long long)b * top_c + js];
-        selS = (selp >= 0 && (long long)selp < t) ? scores[t0 + selp] : 0.f;
+        selS = (tok_ok && selp >= 0 && (long long)selp < t) ? scores[t0 + selp] : 0.f;
     }
     if (st == 0)
         for (int x = tid; x < N * beta; x += kDecThreads)
@@ -546,7 +551,7 @@ accept_decide(const float *__restrict__ logits, int V, const int32_t *__restrict
 
     // ---- outputs of a rejected request ----
     if (st != 0) {
-        for (int i = tid; i < N; i += kDecThreads) {
+        for (int i = tid; rows_ok && i < N; i += kDecThreads) {
             p_tok[n0 + i] = 0.f;
             commit[n0 + i] = 0;
         }
@@ -753,7 +758,7 @@ extern "C" rs_status rs_accept(const float *logits, int R, int V, const int32_t 
         }
     }
     if (B > 0) {
-        launch_pdl(accept_decide, dim3(B), dim3(kDecThreads), 0, st, logits, V, node_off, tokens, parents,
+        launch_pdl(accept_decide, dim3(B), dim3(kDecThreads), 0, st, logits, R, V, node_off, tokens, parents,
             source, chain, sel_pos, tok_off, p, acc_cap, argmax, topk, lse, rowmax, p_tok, acc_len, acc_nodes,
             bonus, winner, commit, scores, status);
         RS_CHECK_LAUNCH("rs_accept/accept_decide");

@@ -33,20 +33,25 @@ namespace {
 
 __global__ void __launch_bounds__(256)
 attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_len,
-          const int32_t *__restrict__ parents, int Hq, int Hkv, int D, ReqInfo *__restrict__ info,
-          uint32_t *__restrict__ anc, float *__restrict__ out, float *__restrict__ lse,
-          int32_t *__restrict__ status) {
+          const int64_t *__restrict__ kv_off, const int32_t *__restrict__ parents, int R, long long kv_rows,
+          int Hq, int Hkv, int D, ReqInfo *__restrict__ info, uint32_t *__restrict__ anc,
+          float *__restrict__ out, float *__restrict__ lse, int32_t *__restrict__ status) {
     pdl_enter();
     const int b = blockIdx.x, tid = threadIdx.x;
     const int n0 = node_off[b];
     const int N = node_off[b + 1] - n0;
     const int S = ctx_len[b];
+    const long long kv0 = kv_off[b];
     const int G = Hq / Hkv;
     __shared__ int s_par[RS_MAX_NODES];
     __shared__ int s_bad;
 
+    // the request's rows must lie in [0, R) and its keys (prefix, then one
+    // slot per node) in [0, kv_rows); outside them nothing is read or written
+    const bool rows_ok = n0 >= 0 && N >= 0 && (long long)n0 + N <= R;
     int st = 0;
-    if (N < 0 || S < 0) st = RS_ST_BAD_TREE;
+    if (!rows_ok || kv0 < 0 || (S >= 0 && kv0 + S + N > kv_rows)) st = RS_ST_BAD_OFFSET;
+    else if (S < 0) st = RS_ST_BAD_TREE;
     else if (N > RS_MAX_NODES) st = RS_ST_TOO_LARGE;
     if (tid == 0) s_bad = 0;
     __syncthreads();
@@ -75,7 +80,7 @@ attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_
         }
     } else {
         if (tid == 0) info[b] = ReqInfo{0, 0, 0, 0};
-        if (N > 0) {
+        if (rows_ok && N > 0) {
             const long long n = (long long)N * Hq;
             for (long long x = tid; x < n * D; x += blockDim.x) out[(long long)n0 * Hq * D + x] = 0.f;
             for (long long x = tid; x < n; x += blockDim.x) lse[(long long)n0 * Hq + x] = 0.f;
@@ -390,7 +395,8 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
         return RS_ERR_CUDA;
     }
 
-    launch_pdl(attn_prep, dim3(B), dim3(256), 0, st, node_off, ctx_len, parents, Hq, Hkv, D, info, anc, out, lse,
+    launch_pdl(attn_prep, dim3(B), dim3(256), 0, st, node_off, ctx_len, kv_off, parents, R, (long long)kv_rows, Hq,
+        Hkv, D, info, anc, out, lse,
         status);
     RS_CHECK_LAUNCH("rs_tree_verify_attn/prep");
 

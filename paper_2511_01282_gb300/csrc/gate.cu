@@ -195,12 +195,16 @@ __device__ __forceinline__ int push_scan(int v, int *s_w, int *total) {
 
 __global__ void __launch_bounds__(kPushThreads)
 gate_push(const float *__restrict__ entropy, const int32_t *__restrict__ row_off,
-          const uint8_t *__restrict__ row_commit, rs_params p, float *__restrict__ hist,
+          const uint8_t *__restrict__ row_commit, int R, rs_params p, float *__restrict__ hist,
           int32_t *__restrict__ hist_n, int32_t *__restrict__ k_star, float *__restrict__ h_best,
           uint8_t *__restrict__ entropy_ok) {
     pdl_enter();
     const int b = blockIdx.x, tid = threadIdx.x;
-    const int r0 = row_off[b], r1 = row_off[b + 1];
+    // rows [r0, r1) must lie in [0, R) (R < 0: the row offsets' last entry);
+    // a range outside them pushes nothing
+    const int rend = R >= 0 ? R : row_off[gridDim.x];
+    int r0 = row_off[b], r1 = row_off[b + 1];
+    if (r0 < 0 || r1 < r0 || r1 > rend) r0 = r1 = 0;
     const int l = p.l;
     __shared__ float s_h[RS_MAX_L];
     __shared__ int s_w[kPushWarps];
@@ -291,7 +295,7 @@ rs_status launch_gate(const char *who, const float *logits, int R, int V, int nc
         RS_CHECK_LAUNCH(who);
     }
     if (B > 0) {
-        launch_pdl(gate_push, dim3(B), dim3(kPushThreads), 0, st, entropy, row_off, row_commit, p, hist, hist_n,
+        launch_pdl(gate_push, dim3(B), dim3(kPushThreads), 0, st, entropy, row_off, row_commit, R, p, hist, hist_n,
             k_star, h_best, entropy_ok);
         RS_CHECK_LAUNCH(who);
     }
@@ -441,8 +445,8 @@ extern "C" rs_status rs_entropy_gate_rows(const float *entropy, const int32_t *r
     RS_CHECK_ARG(B == 0 || (entropy && row_off && row_commit && hist && hist_n && k_star && h_best && entropy_ok),
                  "rs_entropy_gate_rows: null pointer");
     if (B == 0) return RS_OK;
-    launch_pdl(gate_push, dim3(B), dim3(kPushThreads), 0, (cudaStream_t)stream, entropy, row_off, row_commit, p,
-        hist, hist_n, k_star, h_best, entropy_ok);
+    launch_pdl(gate_push, dim3(B), dim3(kPushThreads), 0, (cudaStream_t)stream, entropy, row_off, row_commit, -1,
+        p, hist, hist_n, k_star, h_best, entropy_ok);
     RS_CHECK_LAUNCH("rs_entropy_gate_rows");
     return RS_OK;
 }

@@ -66,6 +66,7 @@ constexpr int kRadixThreads = 256;       // 8 warps x 512 keys per tile
 constexpr int kAppThreads = 256;         // positions per append round
 
 struct IndexView {
+    int32_t *valid;         // 1 when the build's offsets were consistent (else the index holds nothing)
     int64_t *built, *base;  // per request: positions indexed, first list slot
     int32_t *ovf_n;         // per request: overflow entries
     int32_t *start;         // [B][V + 2]
@@ -87,6 +88,7 @@ inline long long n_tiles(long long t_total) { return (t_total + kTile - 1) / kTi
 // Carves the index (and its build scratch) out of `base`; returns the bytes used.
 inline size_t carve_index(void *base, int B, int V, long long t_total, IndexView *v) {
     Carve cv(base);
+    v->valid = cv.take<int32_t>(1);
     v->built = cv.take<int64_t>((size_t)B);
     v->base = cv.take<int64_t>((size_t)B);
     v->ovf_n = cv.take<int32_t>((size_t)B);
@@ -116,10 +118,25 @@ inline int bits_for(long long n) {  // smallest b with n < 2^b
 __device__ __forceinline__ int bucket_of(int tok, int V) { return (tok >= 0 && tok < V) ? tok : V; }
 __device__ __forceinline__ int room_of(int count) { return count + count / 4 + 2; }
 
+// (0) the build's offsets: tok_off[0] = 0, ascending, tok_off[B] = t_total;
+// every later build kernel does nothing unless they are
+__global__ void __launch_bounds__(256)
+index_check(const int64_t *__restrict__ tok_off, int B, long long t_total, IndexView ix) {
+    pdl_enter();
+    __shared__ int s_bad;
+    if (threadIdx.x == 0) s_bad = tok_off[0] != 0 || tok_off[B] != t_total;
+    __syncthreads();
+    for (int b = threadIdx.x; b < B; b += blockDim.x)
+        if (tok_off[b + 1] < tok_off[b]) s_bad = 1;
+    __syncthreads();
+    if (threadIdx.x == 0) *ix.valid = s_bad ? 0 : 1;
+}
+
 // (1) per request: zero the bucket counts, record the request's extent
 __global__ void __launch_bounds__(256)
 index_init(const int64_t *__restrict__ tok_off, int V, IndexView ix) {
     pdl_enter();
+    if (!*ix.valid) return;
     const int b = blockIdx.y;
     const long long stride = (long long)gridDim.x * blockDim.x;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < V + 1; i += stride)
@@ -138,6 +155,7 @@ __global__ void __launch_bounds__(256)
 index_count(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_off, int V, int vbits,
             IndexView ix) {
     pdl_enter();
+    if (!*ix.valid) return;
     const int b = blockIdx.y;
     int32_t *cnt = ix.len + (long long)b * (V + 1);
     const long long t0 = tok_off[b], t = tok_off[b + 1] - t0;
@@ -157,6 +175,7 @@ constexpr int kOffPer = 8;
 __global__ void __launch_bounds__(kIdxThreads)
 index_offsets(int V, IndexView ix) {
     pdl_enter();
+    if (!*ix.valid) return;
     __shared__ int s_w[2][kIdxThreads / 32];
     __shared__ int s_carry[2];
     const int b = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -218,8 +237,10 @@ index_offsets(int V, IndexView ix) {
 
 // (4) radix sort passes: tile histograms ...
 __global__ void __launch_bounds__(kRadixThreads)
-radix_hist(const uint32_t *__restrict__ key, long long N, int shift, long long ntiles, int32_t *__restrict__ hist) {
+radix_hist(const uint32_t *__restrict__ key, long long N, int shift, long long ntiles, int32_t *__restrict__ hist,
+           const int32_t *__restrict__ valid) {
     pdl_enter();
+    if (!*valid) return;
     __shared__ int cnt[kRadixBins];
     const long long tile = blockIdx.x;
     cnt[threadIdx.x] = 0;
@@ -234,8 +255,10 @@ radix_hist(const uint32_t *__restrict__ key, long long N, int shift, long long n
 
 // ... each digit's total over the tiles ...
 __global__ void __launch_bounds__(kRadixThreads)
-radix_total(const int32_t *__restrict__ hist, long long ntiles, int32_t *__restrict__ dtot) {
+radix_total(const int32_t *__restrict__ hist, long long ntiles, int32_t *__restrict__ dtot,
+            const int32_t *__restrict__ valid) {
     pdl_enter();
+    if (!*valid) return;
     __shared__ int s_w[kRadixThreads / 32];
     const int d = blockIdx.x;
     int sum = 0;
@@ -253,8 +276,10 @@ radix_total(const int32_t *__restrict__ hist, long long ntiles, int32_t *__restr
 
 // ... (digit, tile) offsets: the digits below d, then the tiles before t ...
 __global__ void __launch_bounds__(kRadixThreads)
-radix_offsets(int32_t *__restrict__ hist, long long ntiles, const int32_t *__restrict__ dtot) {
+radix_offsets(int32_t *__restrict__ hist, long long ntiles, const int32_t *__restrict__ dtot,
+              const int32_t *__restrict__ valid) {
     pdl_enter();
+    if (!*valid) return;
     __shared__ int s_w[kRadixThreads / 32];
     __shared__ int s_carry;
     const int d = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -292,8 +317,10 @@ radix_offsets(int32_t *__restrict__ hist, long long ntiles, const int32_t *__res
 // the tile (earlier warps, earlier rounds of its warp, lower lanes of its round)
 __global__ void __launch_bounds__(kRadixThreads)
 radix_scatter(const uint32_t *__restrict__ kin, const int32_t *__restrict__ vin, uint32_t *__restrict__ kout,
-              int32_t *__restrict__ vout, long long N, int shift, long long ntiles, const int32_t *__restrict__ hist) {
+              int32_t *__restrict__ vout, long long N, int shift, long long ntiles, const int32_t *__restrict__ hist,
+              const int32_t *__restrict__ valid) {
     pdl_enter();
+    if (!*valid) return;
     constexpr int kWarps = kRadixThreads / 32;
     constexpr int kRounds = kTile / kRadixThreads;
     __shared__ int wcnt[kWarps][kRadixBins];
@@ -345,6 +372,7 @@ __global__ void __launch_bounds__(256)
 index_place(const uint32_t *__restrict__ key, const int32_t *__restrict__ val, long long N,
             const int64_t *__restrict__ tok_off, int V, int vbits, IndexView ix) {
     pdl_enter();
+    if (!*ix.valid) return;
     const long long stride = (long long)gridDim.x * blockDim.x;
     const uint32_t vmask = (vbits >= 32) ? 0xffffffffu : ((1u << vbits) - 1u);
     for (long long j = blockIdx.x * (long long)blockDim.x + threadIdx.x; j < N; j += stride) {
@@ -371,6 +399,12 @@ index_append(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok
     __shared__ int s_novf;
     const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const long long t0 = tok_off[b], t = tok_off[b + 1] - t0;
+    // an index whose build saw inconsistent offsets holds nothing, and the
+    // buffers hold tok_off[B] tokens: otherwise nothing is read or written
+    if (!*ix.valid || t0 < 0 || t < 0 || t0 + t > tok_off[gridDim.x]) {
+        if (tid == 0 && status) status[b] = RS_ST_BAD_OFFSET;
+        return;
+    }
     const int32_t *X = tokens + t0;
     int32_t *start = ix.start + (long long)b * (V + 2);
     int32_t *len = ix.len + (long long)b * (V + 1);
@@ -468,11 +502,14 @@ index_query(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_
     const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const long long t0 = tok_off[b];
     const long long t = tok_off[b + 1] - t0;
-    const int32_t *X = tokens + t0;
-    const float *S = scores + t0;
+    // an index whose build saw inconsistent offsets holds nothing, and the
+    // buffers hold tok_off[B] tokens: otherwise the request is not read
+    const bool off_ok = *ix.valid && t0 >= 0 && t >= 0 && t0 + t <= tok_off[gridDim.x];
+    const int32_t *X = tokens + (off_ok ? t0 : 0);
+    const float *S = scores + (off_ok ? t0 : 0);
     const int k = k_star[b];
-    int st = 0;
-    bool run = k > 0 && (gate_ok == nullptr || gate_ok[b] != 0);
+    int st = off_ok ? 0 : RS_ST_BAD_OFFSET;
+    bool run = off_ok && k > 0 && (gate_ok == nullptr || gate_ok[b] != 0);
     if (run && k > RS_MAX_L) {
         st = RS_ST_TOO_LARGE;
         run = false;
@@ -702,6 +739,8 @@ extern "C" rs_status rs_match_index_build(const int32_t *tokens, const int64_t *
     carve_index(index, B, V, t_total, &ix);
     const int vbits = bits_for(V);
     const int keybits = vbits + bits_for(B - 1);
+    launch_pdl(index_check, dim3(1), dim3(256), 0, st, tok_off, B, (long long)t_total, ix);
+    RS_CHECK_LAUNCH("rs_match_index_build/check");
     const unsigned zx = (unsigned)std::min<long long>((V + 1 + 255) / 256, 64);
     launch_pdl(index_init, dim3(zx, B), dim3(256), 0, st, tok_off, V, ix);
     RS_CHECK_LAUNCH("rs_match_index_build/init");
@@ -715,14 +754,15 @@ extern "C" rs_status rs_match_index_build(const int32_t *tokens, const int64_t *
     const long long N = t_total, nt = n_tiles(t_total);
     int cur = 0;
     for (int shift = 0; shift < keybits; shift += 8, cur ^= 1) {
-        launch_pdl(radix_hist, dim3((unsigned)nt), dim3(kRadixThreads), 0, st, ix.key[cur], N, shift, nt, ix.hist);
+        launch_pdl(radix_hist, dim3((unsigned)nt), dim3(kRadixThreads), 0, st, ix.key[cur], N, shift, nt, ix.hist,
+                   ix.valid);
         RS_CHECK_LAUNCH("rs_match_index_build/radix_hist");
-        launch_pdl(radix_total, dim3(kRadixBins), dim3(kRadixThreads), 0, st, ix.hist, nt, ix.dtot);
+        launch_pdl(radix_total, dim3(kRadixBins), dim3(kRadixThreads), 0, st, ix.hist, nt, ix.dtot, ix.valid);
         RS_CHECK_LAUNCH("rs_match_index_build/radix_total");
-        launch_pdl(radix_offsets, dim3(kRadixBins), dim3(kRadixThreads), 0, st, ix.hist, nt, ix.dtot);
+        launch_pdl(radix_offsets, dim3(kRadixBins), dim3(kRadixThreads), 0, st, ix.hist, nt, ix.dtot, ix.valid);
         RS_CHECK_LAUNCH("rs_match_index_build/radix_offsets");
         launch_pdl(radix_scatter, dim3((unsigned)nt), dim3(kRadixThreads), 0, st, ix.key[cur], ix.val[cur],
-                   ix.key[cur ^ 1], ix.val[cur ^ 1], N, shift, nt, ix.hist);
+                   ix.key[cur ^ 1], ix.val[cur ^ 1], N, shift, nt, ix.hist, ix.valid);
         RS_CHECK_LAUNCH("rs_match_index_build/radix_scatter");
     }
     const unsigned px = (unsigned)std::min<long long>((N + 255) / 256, 148ll * 16);

@@ -297,7 +297,7 @@ sample_pick(const float *__restrict__ logits, int V, int nchunks, float scale, c
 
 // One warp per request: the tree check and the walk along model children.
 __global__ void __launch_bounds__(32)
-sample_walk(const int32_t *__restrict__ node_off, const int32_t *__restrict__ tokens,
+sample_walk(const int32_t *__restrict__ node_off, int R, const int32_t *__restrict__ tokens,
             const int32_t *__restrict__ parents, const uint8_t *__restrict__ source,
             const int32_t *__restrict__ draw, int acc_cap, int32_t *__restrict__ acc_len,
             int32_t *__restrict__ acc_nodes, int32_t *__restrict__ bonus, int32_t *__restrict__ status) {
@@ -309,7 +309,8 @@ sample_walk(const int32_t *__restrict__ node_off, const int32_t *__restrict__ to
     int32_t *an = acc_nodes + (long long)b * acc_cap;
     for (int j = lane; j < acc_cap; j += 32) an[j] = -1;
     int st = 0;
-    if (N > RS_MAX_NODES) st = RS_ST_TOO_LARGE;
+    if (n0 < 0 || N < 0 || (long long)n0 + N > R) st = RS_ST_BAD_OFFSET;  // rows outside [0, R): not read
+    else if (N > RS_MAX_NODES) st = RS_ST_TOO_LARGE;
     else if (N < 1) st = RS_ST_BAD_TREE;
     // node i = lane + 32 q lives in register slot q
     int par[kPer], tok[kPer];
@@ -411,7 +412,7 @@ extern "C" rs_status rs_tree_sample(const float *logits, int R, int V, const int
         RS_CHECK_LAUNCH("rs_tree_sample/pick");
     }
     if (B > 0) {
-        launch_pdl(sample_walk, dim3(B), dim3(32), 0, st, node_off, tokens, parents, source, draw, acc_cap, acc_len,
+        launch_pdl(sample_walk, dim3(B), dim3(32), 0, st, node_off, R, tokens, parents, source, draw, acc_cap, acc_len,
             acc_nodes, bonus, status);
         RS_CHECK_LAUNCH("rs_tree_sample/walk");
     }

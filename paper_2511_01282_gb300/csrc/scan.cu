@@ -208,12 +208,14 @@ match_scan_kernel(const int32_t *__restrict__ tokens, const int64_t *__restrict_
     ScanShared &sh = *reinterpret_cast<ScanShared *>(scan_smem);
     const long long t0 = tok_off[b];
     const long long t = tok_off[b + 1] - t0;
-    const int32_t *X = tokens + t0;
-    const float *S = scores + t0;
+    // the buffers hold tok_off[B] tokens: a range outside them is not read
+    const bool off_ok = t0 >= 0 && t >= 0 && t0 + t <= tok_off[gridDim.y];
+    const int32_t *X = tokens + (off_ok ? t0 : 0);
+    const float *S = scores + (off_ok ? t0 : 0);
     const int k = k_star[b];
 
-    int st = 0;
-    bool run = k > 0 && (gate_ok == nullptr || gate_ok[b] != 0);
+    int st = off_ok ? 0 : RS_ST_BAD_OFFSET;
+    bool run = off_ok && k > 0 && (gate_ok == nullptr || gate_ok[b] != 0);
     if (run && k > RS_MAX_L) {
         st = RS_ST_TOO_LARGE;
         run = false;

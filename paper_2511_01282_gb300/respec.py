@@ -17,6 +17,7 @@ LIB_PATH = os.path.join(_HERE, "librespec.so")
 
 RS_OK, RS_ERR_INVALID_ARG, RS_ERR_UNSUPPORTED, RS_ERR_CAPACITY, RS_ERR_CUDA = range(5)
 RS_ST_BAD_TREE, RS_ST_TRUNCATED, RS_ST_BAD_POS, RS_ST_TOO_LARGE, RS_ST_TIMEOUT = 1, 2, 4, 8, 16
+RS_ST_BAD_OFFSET = 32
 RS_MAX_L, RS_MAX_TOPC, RS_MAX_SPAN, RS_MAX_BETA, RS_MAX_NODES = 8, 8, 256, 16, 256
 
 

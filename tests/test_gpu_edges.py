@@ -322,3 +322,129 @@ def test_scan_long_buffers(dense):
     for key in ("count", "pos", "sel_pos", "sel_len", "spans", "n_sel", "status"):
         assert (got[key] == ref[key]).all(), key
     assert (ref["n_sel"] > 0).all()
+
+
+# ------------------------------------------------------------------ offsets out of bounds
+# Offsets arrays are device data the host cannot check: every kernel checks the
+# ranges it reads before indexing with them.  Requests 1 and 2 get ranges that
+# run past the arrays (past R, kv_rows or the buffers' tok_off[B] tokens, or a
+# negative length); they are reported RS_ST_BAD_OFFSET and skipped, and
+# request 0 (same range as in the valid workload) still matches the oracle.
+BIG = 1 << 28
+
+
+def _bad_offsets(off):
+    """off[B+1] with request 1's end and request 2's start far past the end."""
+    bad = np.array(off, dtype=np.int64).copy()
+    bad[2] = BIG
+    return bad
+
+
+def test_attention_offsets_out_of_bounds():
+    w = synth.build(synth.small_spec(B=3, V=500), seed=21)
+    s = w.spec
+    st = make_step(w)
+    node_off = _bad_offsets(w.node_off).astype(np.int32)
+    st.d["node_off"] = _cuda(node_off)
+    st.attn()
+    torch.cuda.synchronize()
+    status = host(st.out["attn_status"])
+    assert status[0] == 0 and status[1] == rs.RS_ST_BAD_OFFSET and status[2] == rs.RS_ST_BAD_OFFSET
+    n0, n1 = int(w.node_off[0]), int(w.node_off[1])
+    rows = [(n, h) for n in range(n0, n1) for h in range(s.Hq)]
+    ref = oracle.tree_attn(w.q, w.k, w.v, w.kv_off, w.ctx_len, w.node_off, w.parents, s.Hq, s.Hkv, s.D,
+                           st.scale, rows=rows)
+    got = host(st.out["attn_out"])[n0:n1].reshape(-1, s.D)
+    assert np.abs(got - ref["out"]).max() < 1e-2
+    # keys past kv_rows: request 2's prefix ends beyond the KV cache
+    st = make_step(w)
+    kv_off = w.kv_off.copy()
+    kv_off[2] = st.kv_rows - 1
+    st.d["kv_off"] = _cuda(kv_off)
+    st.attn()
+    torch.cuda.synchronize()
+    assert host(st.out["attn_status"]).tolist() == [0, 0, rs.RS_ST_BAD_OFFSET]
+
+
+def test_accept_and_sample_offsets_out_of_bounds():
+    w = synth.build(synth.small_spec(B=3, V=700), seed=22)
+    s = w.spec
+    ref = oracle.accept(w.logits, w.node_off, w.tree_tokens, w.parents, w.source, w.chain, w.sel_pos,
+                        w.tok_off, w.scores, s.beta, f32(s.tau), s.phi, s.m, f32(s.alpha), 64)
+    st = make_step(w)
+    st.d["node_off"] = _cuda(_bad_offsets(w.node_off).astype(np.int32))
+    st.accept()
+    torch.cuda.synchronize()
+    o = st.out
+    stt = host(o["acc_status"])
+    assert stt[0] == ref["status"][0] and stt[1] == rs.RS_ST_BAD_OFFSET and stt[2] == rs.RS_ST_BAD_OFFSET
+    for k in ("acc_len", "bonus", "winner"):
+        assert host(o[k])[0] == ref[k][0], k
+    assert (host(o["acc_nodes"])[0] == ref["acc_nodes"][0]).all()
+    assert (host(o["winner"])[1:] == -2).all() and (host(o["acc_len"])[1:] == 0).all()
+    # the score table: request 0's selected positions updated as the oracle's, the rest untouched
+    t1 = int(w.tok_off[1])
+    assert (host(st.d["scores"])[:t1] == ref["scores"][:t1]).all()
+    assert (host(st.d["scores"])[t1:] == w.scores[t1:]).all()
+    # tok_off past the score table for request 1
+    st = make_step(w)
+    tok_off = w.tok_off.copy()
+    tok_off[2] = tok_off[3] + 5
+    st.d["tok_off"] = _cuda(tok_off)
+    st.accept()
+    torch.cuda.synchronize()
+    assert host(st.out["acc_status"])[1] & rs.RS_ST_BAD_OFFSET
+    # sampling walk
+    st = make_step(w)
+    st.d["node_off"] = _cuda(_bad_offsets(w.node_off).astype(np.int32))
+    st.tree_sample(1.0)
+    torch.cuda.synchronize()
+    so = {k: host(v) for k, v in st.sample_out.items()}
+    assert so["status"][1] == rs.RS_ST_BAD_OFFSET and so["status"][2] == rs.RS_ST_BAD_OFFSET
+    assert so["acc_len"][1] == 0 and so["bonus"][1] == -1
+
+
+def test_scan_gate_and_index_offsets_out_of_bounds():
+    w = synth.build(synth.small_spec(B=3, V=300, repeat_prob=0.6, seg_len=(3, 8)), seed=23)
+    s = w.spec
+    ks = np.array([2, 2, 2], np.int32)
+    tok_bad = _bad_offsets(w.tok_off)
+    tok_bad[-1] = w.tok_off[-1]              # the buffers hold tok_off[B] tokens
+    ref = oracle.match_scan(w.tokens, w.tok_off, ks, w.scores, f32(s.theta_score), s.top_c, s.chain_len,
+                            s.pos_cap)
+    st = make_step(w)
+    st.d["tok_off"] = _cuda(tok_bad)
+    st.scan(k_star=_cuda(ks), gate_ok=None)
+    torch.cuda.synchronize()
+    o = st.out
+    assert host(o["scan_status"]).tolist()[1:] == [rs.RS_ST_BAD_OFFSET] * 2
+    for k_gpu, k_ref in (("count", "count"), ("pos", "pos"), ("sel_pos", "sel_pos"), ("spans", "spans")):
+        assert (host(o[k_gpu])[0] == ref[k_ref][0]).all(), k_gpu
+    assert (host(o["n_sel"])[1:] == 0).all()
+    # the trigger: a request whose rows run past the entropies pushes nothing
+    st = make_step(w)
+    row_bad = _bad_offsets(w.node_off).astype(np.int32)
+    st.d["row_off"] = _cuda(row_bad)
+    st.out["acc_entropy"].copy_(torch.from_numpy(oracle.entropy_rows(w.logits).astype(np.float32)))
+    st.gate_rows()
+    torch.cuda.synchronize()
+    H = host(st.out["acc_entropy"]).astype(np.float64)
+    off0 = np.array([0, w.node_off[1], w.node_off[1], w.node_off[1]], np.int64)  # rows of request 0 only
+    g = oracle.gate(H, off0, w.row_commit, w.hist, w.hist_n, s.l, f32(s.lambda_e), f32(s.theta_entropy))
+    assert (host(st.out["k_star"]) == g["k_star"]).all() and (host(st.d["hist"]) == g["hist"].astype(np.float32)).all()
+    # the index: a build on inconsistent offsets holds nothing; a query with a
+    # request out of bounds skips it
+    from test_gpu_index import build_index, query
+    idx, t_total = build_index(w.tokens, tok_bad, s.V)
+    got = query(w.tokens, w.tok_off, ks, None, w.scores, s.theta_score, s.top_c, s.chain_len, 16, s.V, t_total, idx)
+    assert (got["status"] == rs.RS_ST_BAD_OFFSET).all()
+    status = torch.zeros(3, dtype=torch.int32, device="cuda")
+    rs.rs_match_index_append(_cuda(w.tokens), _cuda(w.tok_off), 3, s.V, t_total, idx, status)
+    torch.cuda.synchronize()
+    assert (host(status) == rs.RS_ST_BAD_OFFSET).all()
+    idx, t_total = build_index(w.tokens, w.tok_off, s.V)
+    got = query(w.tokens, tok_bad, ks, None, w.scores, s.theta_score, s.top_c, s.chain_len, 16, s.V, t_total, idx)
+    ref16 = oracle.match_scan(w.tokens, w.tok_off, ks, w.scores, f32(s.theta_score), s.top_c, s.chain_len, 16)
+    assert got["status"].tolist()[1:] == [rs.RS_ST_BAD_OFFSET] * 2
+    for k in ("count", "pos", "sel_pos", "spans"):
+        assert (got[k][0] == ref16[k][0]).all(), k
