@@ -382,10 +382,17 @@ rs_status rs_match_scan_indexed(const int32_t *tokens, const int64_t *tok_off, i
  *   status  [B] int32     RS_ST_BAD_TREE (parents / source layout) or
  *                         RS_ST_TOO_LARGE (more than RS_MAX_NODES nodes):
  *                         acc_len 0, bonus -1.
+ * Draws are exact: each is the fp64 inverse CDF above (exp and sums in fp64,
+ * token-id order), up to rounding at the 1e-12 level of Z.  An fp32 pass
+ * settles each row under a rigorous error bound; rows whose u Z lies within
+ * that bound of a CDF step (a few percent of high-entropy rows) are redone
+ * in double-float arithmetic, spread over the GPU.
  * Workspace: rs_tree_sample_workspace_size(R, V) bytes (per 8192-logit chunk
- * of every row: its maximum and its mass).  Draws are computed in fp32; a
- * uniform within ~1e-5 relative of a CDF step may land on the neighbouring
- * token relative to an fp64 evaluation.
+ * of every row its maximum and mass terms; the list of redone rows; per
+ * 512-id slice of every row a double-float sum).  Stream-ordered: a call
+ * must not share its workspace with a call in flight on another stream.
+ * Environment: RS_DEBUG_SAMPLE_EXACT=1 (a test hook) redoes every row with
+ * mass.
  */
 size_t rs_tree_sample_workspace_size(int R, int V);
 rs_status rs_tree_sample(const float *logits, int R, int V, const int32_t *node_off, int B,
