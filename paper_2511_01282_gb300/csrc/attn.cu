@@ -22,10 +22,12 @@
 
 #include <algorithm>
 #include <cstdlib>
+#include <cstring>
 
 #include <mutex>
 
 #include "attn_core.cuh"
+#include "attn_pair.cuh"
 #include "common.cuh"
 
 namespace rs {
@@ -34,7 +36,7 @@ namespace {
 __global__ void __launch_bounds__(256)
 attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_len,
           const int64_t *__restrict__ kv_off, const int32_t *__restrict__ parents, int R, long long kv_rows,
-          int Hq, int Hkv, int D, ReqInfo *__restrict__ info, uint32_t *__restrict__ anc,
+          int Hq, int Hkv, int D, int seg_rows, ReqInfo *__restrict__ info, uint32_t *__restrict__ anc,
           float *__restrict__ out, float *__restrict__ lse, int32_t *__restrict__ status) {
     pdl_enter();
     const int b = blockIdx.x, tid = threadIdx.x;
@@ -74,9 +76,9 @@ attn_prep(const int32_t *__restrict__ node_off, const int32_t *__restrict__ ctx_
             for (int w = 0; w < kAncWords; ++w) anc[(long long)(n0 + i) * kAncWords + w] = bits[w];
         }
         if (tid == 0) {
-            int mt = (N * G + kBM - 1) / kBM;
+            int mt = (N * G + seg_rows - 1) / seg_rows;
             int nt = (S + N + kBN - 1) / kBN;
-            info[b] = ReqInfo{Hkv * mt * nt, mt, nt, 1};
+            info[b] = ReqInfo{Hkv * mt * nt, mt, nt, N * G};
         }
     } else {
         if (tid == 0) info[b] = ReqInfo{0, 0, 0, 0};
@@ -137,8 +139,8 @@ __device__ __forceinline__ void combine_item(const AttnArgs &a, const CombJob &j
     const int q = lane % kLpr;
     const int grp = (int)(threadIdx.x >> 5) * kSub + lane / kLpr;
     const int G = a.Hq / a.Hkv;
-    const int rows = min(kBM, job.N * G - job.mtile * kBM);
-    const int rbase = row0 + grp * rpw;                 // this lane's first row in the tile
+    const int rows = min(a.seg_rows, job.N * G - job.mtile * a.seg_rows);
+    const int rbase = row0 + grp * rpw;                 // this lane's first row in the segment
     const int npairs = max(0, min(rpw, rows - rbase)) * np;
     // piece p > 0: slot 0 of the p-th CTA with a non-empty range after CTA c
     auto slot_of = [&](int p) -> long long { return p == 0 ? job.first_slot : 2ll * nonempty[p]; };
@@ -156,7 +158,7 @@ __device__ __forceinline__ void combine_item(const AttnArgs &a, const CombJob &j
                 l[s] = 0.f;
                 o[s] = make_float4(0.f, 0.f, 0.f, 0.f);
                 if (x0 + s < npairs) {
-                    const long long prow = slot_of(pp) * kBM + rbase + kk;
+                    const long long prow = slot_of(pp) * a.seg_rows + rbase + kk;
                     m[s] = a.part_m[prow];
                     l[s] = a.part_l[prow];
                     o[s] = *reinterpret_cast<const float4 *>(a.part_o + prow * D + q * 4);
@@ -186,7 +188,7 @@ __device__ __forceinline__ void combine_item(const AttnArgs &a, const CombJob &j
                 }
             }
             if (++p == np) {  // row rbase + k complete
-                const int rr = job.mtile * kBM + rbase + k;
+                const int rr = job.mtile * a.seg_rows + rbase + k;
                 const int i = rr / G, h = job.kvh * G + (rr - i * G);
                 const long long orow = (long long)(job.n0 + i) * a.Hq + h;
                 const float f = L > 0.f ? 1.f / L : 0.f;
@@ -246,7 +248,7 @@ attn_combine(AttnArgs a, int Gc) {
     if (t < Gc && j.b >= 0) {
         const int np = s_rank[j.c1] - rank + 1;  // CTAs t and c1 both hold a piece
         const int rpw = np <= 2 ? 4 : (np <= 4 ? 2 : 1);
-        const int rows = min(kBM, j.N * G - j.mtile * kBM);
+        const int rows = min(a.seg_rows, j.N * G - j.mtile * a.seg_rows);
         const int per = rows_per_group * rpw;
         s_np[t] = np;
         s_rpw[t] = rpw;
@@ -299,7 +301,25 @@ bool make_kv_map(CUtensorMap *m, const void *base, long long kv_rows, int Hkv, i
     return r == CUDA_SUCCESS;
 }
 
-int g_attr_done[64][2] = {};
+int g_attr_done[64][2] = {};       // one-tile form, per device and head dim
+int g_pair_attr_done[64][2] = {};  // two-tile form
+int g_pair_regs_ok[64][2] = {};    // two-tile form: 1 usable, -1 not (register budget)
+
+// Rows per segment: 256 selects the two-row-tile form (attn_pair.cuh), which
+// pays off when requests have more than one 128-row tile per KV head.  The
+// host cannot see the trees, so it judges from the average over the call:
+// more (node, q-head-in-group) rows per request and KV head than one tile.
+// RS_DEBUG_ATTN_FORM=one|pair overrides the choice (a test hook: both forms
+// compute the same function).
+int attn_seg_rows(int B, int R, int Hq, int Hkv, int D) {
+    const bool pair_ok = B <= kPairMaxB;
+    if (const char *e = getenv("RS_DEBUG_ATTN_FORM")) {
+        if (!strcmp(e, "pair")) return pair_ok ? kPairRows : kBM;
+        if (!strcmp(e, "one")) return kBM;
+    }
+    const long long G = Hkv > 0 ? Hq / Hkv : 1;
+    return (pair_ok && D == 128 && (long long)R * G > (long long)kBM * B) ? kPairRows : kBM;
+}
 
 }  // namespace
 }  // namespace rs
@@ -311,12 +331,13 @@ static int attn_grid() { return std::min(num_sms(), kAttnMaxGrid); }
 extern "C" size_t rs_tree_verify_attn_workspace_size(int B, int R, int Hq, int Hkv, int D) {
     if (B < 0 || R < 0 || Hq < 1 || Hkv < 1 || (D != 64 && D != 128)) return 0;
     const size_t Gc = (size_t)attn_grid();
+    const size_t rows = (size_t)attn_seg_rows(B, R, Hq, Hkv, D);
     Carve cv(nullptr);
     cv.take<ReqInfo>((size_t)B);
     cv.take<uint32_t>((size_t)R * kAncWords);
-    cv.take<float>(2 * Gc * kBM * (size_t)D);
-    cv.take<float>(2 * Gc * kBM);
-    cv.take<float>(2 * Gc * kBM);
+    cv.take<float>(2 * Gc * rows * (size_t)D);
+    cv.take<float>(2 * Gc * rows);
+    cv.take<float>(2 * Gc * rows);
     cv.take<CombJob>(Gc);
     cv.take<int2>(Gc);
     return cv.used();
@@ -354,6 +375,7 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
         return RS_ERR_CAPACITY;
     }
     const int Gc = attn_grid();
+    const int seg_rows = attn_seg_rows(B, R, Hq, Hkv, D);
     Carve cv(workspace);
     ReqInfo *info = cv.take<ReqInfo>((size_t)B);
     uint32_t *anc = cv.take<uint32_t>((size_t)R * kAncWords);
@@ -363,9 +385,10 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     a.ctx_len = ctx_len;
     a.node_off = node_off;
     a.anc = anc;
-    a.part_o = cv.take<float>(2 * (size_t)Gc * kBM * D);
-    a.part_m = cv.take<float>(2 * (size_t)Gc * kBM);
-    a.part_l = cv.take<float>(2 * (size_t)Gc * kBM);
+    a.part_o = cv.take<float>(2 * (size_t)Gc * seg_rows * D);
+    a.part_m = cv.take<float>(2 * (size_t)Gc * seg_rows);
+    a.part_l = cv.take<float>(2 * (size_t)Gc * seg_rows);
+    a.seg_rows = seg_rows;
     a.jobs = cv.take<CombJob>((size_t)Gc);
     a.ranges = cv.take<int2>((size_t)Gc);
     a.B = B;
@@ -395,31 +418,64 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
         return RS_ERR_CUDA;
     }
 
-    launch_pdl(attn_prep, dim3(B), dim3(256), 0, st, node_off, ctx_len, kv_off, parents, R, (long long)kv_rows, Hq,
-        Hkv, D, info, anc, out, lse,
-        status);
-    RS_CHECK_LAUNCH("rs_tree_verify_attn/prep");
-
     int dev = 0;
     cudaGetDevice(&dev);
     const int di = D == 128 ? 1 : 0;
-    const size_t smem_max = attn_smem_bytes(kAttnMaxB);
-    if (dev >= 0 && dev < 64 && !g_attr_done[dev][di]) {
-        cudaError_t e = D == 128 ? cudaFuncSetAttribute(attn_tc_kernel<128>,
-                                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_max)
-                                 : cudaFuncSetAttribute(attn_tc_kernel<64>,
-                                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_max);
+    const bool pair = seg_rows == kPairRows;
+    if (pair && dev >= 0 && dev < 64 && g_pair_regs_ok[dev][di] == 0) {
+        // The two-tile kernel moves registers between its warpgroups with
+        // setmaxnreg, sized for a launch of 168 registers per thread; with
+        // fewer at launch the raise could never be granted.  Checked once.
+        cudaFuncAttributes fa;
+        const cudaError_t e = D == 128 ? cudaFuncGetAttributes(&fa, attn_pair_kernel<128>)
+                                       : cudaFuncGetAttributes(&fa, attn_pair_kernel<64>);
+        g_pair_regs_ok[dev][di] = (e == cudaSuccess && fa.numRegs * kPairThreads >=
+                                   (int)(2 * 128 * kPairRegsSoft + 128 * kPairRegsProd)) ? 1 : -1;
+    }
+    if (pair && (dev < 0 || dev >= 64 || g_pair_regs_ok[dev][di] != 1)) {
+        set_error("rs_tree_verify_attn: two-tile kernel built with too few registers per thread");
+        return RS_ERR_CUDA;
+    }
+    launch_pdl(attn_prep, dim3(B), dim3(256), 0, st, node_off, ctx_len, kv_off, parents, R, (long long)kv_rows, Hq,
+        Hkv, D, seg_rows, info, anc, out, lse,
+        status);
+    RS_CHECK_LAUNCH("rs_tree_verify_attn/prep");
+
+    int(&attr_done)[64][2] = pair ? g_pair_attr_done : g_attr_done;
+    if (dev >= 0 && dev < 64 && !attr_done[dev][di]) {
+        cudaError_t e;
+        if (pair) {
+            const int smem_max = (int)attn_pair_smem_bytes(kPairMaxB);
+            e = D == 128 ? cudaFuncSetAttribute(attn_pair_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                smem_max)
+                         : cudaFuncSetAttribute(attn_pair_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                smem_max);
+        } else {
+            const int smem_max = (int)attn_smem_bytes(kAttnMaxB);
+            e = D == 128 ? cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                smem_max)
+                         : cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                smem_max);
+        }
         if (e != cudaSuccess) {
             set_error("rs_tree_verify_attn: cudaFuncSetAttribute: %s", cudaGetErrorString(e));
             return RS_ERR_CUDA;
         }
-        g_attr_done[dev][di] = 1;
+        attr_done[dev][di] = 1;
     }
-    const size_t smem = attn_smem_bytes(B);
-    if (D == 128)
-        launch_full(attn_tc_kernel<128>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
-    else
-        launch_full(attn_tc_kernel<64>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
+    if (pair) {
+        const size_t smem = attn_pair_smem_bytes(B);
+        if (D == 128)
+            launch_full(attn_pair_kernel<128>, dim3(Gc), dim3(kPairThreads), smem, st, a, info, tmk, tmv);
+        else
+            launch_full(attn_pair_kernel<64>, dim3(Gc), dim3(kPairThreads), smem, st, a, info, tmk, tmv);
+    } else {
+        const size_t smem = attn_smem_bytes(B);
+        if (D == 128)
+            launch_full(attn_tc_kernel<128>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
+        else
+            launch_full(attn_tc_kernel<64>, dim3(Gc), dim3(kAttnThreads), smem, st, a, info, tmk, tmv);
+    }
     RS_CHECK_LAUNCH("rs_tree_verify_attn/main");
     // a full launch: combine blocks parked early beside the attention CTAs
     // (programmatic launch) measured slower on the batched workload

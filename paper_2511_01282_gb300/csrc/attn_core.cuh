@@ -75,9 +75,9 @@ inline size_t attn_smem_bytes(int B) { return 1024 + kSmemPref + 2 * (size_t)(B 
 
 struct ReqInfo {
     int units;  // Hkv * mt * nt, 0 for a rejected request
-    int mt;     // row tiles
+    int mt;     // row tiles (row-tile pairs in the two-tile form) per KV head
     int nt;     // KV tiles
-    int ok;
+    int rows;   // (node, q-head-in-group) rows per KV head: N * Hq / Hkv
 };
 
 // The split segment a CTA starts, for attn_combine: the segment that begins
@@ -101,6 +101,7 @@ struct AttnArgs {
     CombJob *jobs;  // [gridDim.x]
     int2 *ranges;   // [gridDim.x]: each CTA's unit range [x, y)
     int kv_stream;  // the launch's K/V is large next to L2: stream tiles read once
+    int seg_rows;   // rows per segment and per partial slot: 128, or 256 in the two-tile form
     long long wait_limit;  // clock cycles a pipeline wait may take before the CTA gives up
     int B, Hq, Hkv, D;
     float scale;
