@@ -243,7 +243,13 @@ rs_status rs_match_scan(const int32_t *tokens, const int64_t *tok_off, int B,
  *            workspace must be 16-byte aligned.
  *   status   [B]: RS_ST_BAD_TREE / RS_ST_TOO_LARGE for a malformed request
  *            (its out/lse rows are zeroed).
- * QK^T and PV run on the tensor cores with fp32 accumulation.
+ * QK^T and PV run on the tensor cores with fp32 accumulation.  The call
+ * picks one of two kernel forms from its sizes (one 128-row tile per work
+ * segment, or a pair of tiles sharing each K/V tile when the requests
+ * average more than 128 (node, q-head-in-group) rows per KV head); the
+ * workspace size depends on that choice, so size it with the same five
+ * sizes as the call.  Environment: RS_DEBUG_ATTN_FORM=one|pair (a test
+ * hook) forces either form; both compute the same function.
  */
 size_t rs_tree_verify_attn_workspace_size(int B, int R, int Hq, int Hkv, int D);
 rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, const uint16_t *v,

@@ -465,6 +465,14 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
                     const int jt = pc.j0 + tl;
                     const int b = full ? x : (tl & 1);
                     const uint32_t par = full ? ((b ? use1 : use0) + tl) & 1 : ((b ? use1 : use0) + (tl >> 1)) & 1;
+                    const int key0 = jt * kBN;
+                    const bool masked = key0 + kBN > S;
+                    // the row's ancestor set, for a tile with tree slots: loaded
+                    // before the wait for S so that the wait covers its latency
+                    uint32_t anc[kAncWords];
+#pragma unroll
+                    for (int w = 0; w < kAncWords; ++w)
+                        anc[w] = (valid && masked) ? a.anc[(long long)(n0 + i) * kAncWords + w] : 0u;
                     if (!(ok = warp_wait(&sfull[b], par, s_abort, a.wait_limit))) break;
                     tc_fence_after();
                     // every S reading K of this tile is complete (in full mode S_A
@@ -492,15 +500,10 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
                         }
                     }
                     float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-                    const int key0 = jt * kBN;
-                    if (key0 + kBN <= S) {  // prefix-only: nothing to mask
+                    if (!masked) {  // prefix-only: nothing to mask
 #pragma unroll
                         for (int j = 0; j < kBN; ++j) mx4[j & 3] = fmaxf(mx4[j & 3], s[j]);
                     } else {  // tree slots in this tile: the row's ancestor set decides
-                        uint32_t anc[kAncWords];
-#pragma unroll
-                        for (int w = 0; w < kAncWords; ++w)
-                            anc[w] = valid ? a.anc[(long long)(n0 + i) * kAncWords + w] : 0u;
 #pragma unroll
                         for (int ch = 0; ch < kBN / 32; ++ch) {
                             const uint32_t msk = tree_window(anc, key0 + ch * 32 - S);
@@ -568,25 +571,39 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
                     ok = warp_wait(&vempty[pv & 1], (pv >> 1) & 1, s_abort, a.wait_limit);
                 }
                 if (ok) {
+                    // O rows leave through shared memory (this tile's Q buffer:
+                    // every S of the piece has completed), so that each store
+                    // instruction writes whole 128-byte lines: a warp stages 32
+                    // rows x 32 columns (row stride 36 floats, conflict-free
+                    // both ways) and then writes 4 rows x 32 columns per store.
                     tc_fence_after();
                     const long long orow = (long long)(n0 + i) * a.Hq + h;
                     const long long prow = (long long)pc.slot * kPairRows + x * kBM + r;
                     const float f = pc.final ? ((l > 0.f) ? 1.f / l : 0.f) : 1.f;
-#pragma unroll
+                    float *dst = pc.final ? a.out + orow * D : a.part_o + prow * D;
+                    const unsigned vmask = __ballot_sync(0xffffffffu, valid);
+                    float *stage = reinterpret_cast<float *>(qs + (warp & 3) * 8192);
+#pragma unroll 1
                     for (int ch = 0; ch < D / 32; ++ch) {
                         uint32_t xo[32];
                         tmem_ld32(tmem + lane_off + (uint32_t)x * 128 + ch * 32, xo);
                         tmem_wait_ld();
                         tmem_regs_ready(xo);
-                        if (valid) {
-                            float4 *dst = pc.final ? reinterpret_cast<float4 *>(a.out + orow * D + ch * 32)
-                                                   : reinterpret_cast<float4 *>(a.part_o + prow * D + ch * 32);
 #pragma unroll
-                            for (int e = 0; e < 8; ++e)
-                                dst[e] = make_float4(__uint_as_float(xo[4 * e]) * f, __uint_as_float(xo[4 * e + 1]) * f,
-                                                     __uint_as_float(xo[4 * e + 2]) * f,
-                                                     __uint_as_float(xo[4 * e + 3]) * f);
+                        for (int e = 0; e < 8; ++e)
+                            *reinterpret_cast<float4 *>(stage + lane * 36 + 4 * e) =
+                                make_float4(__uint_as_float(xo[4 * e]) * f, __uint_as_float(xo[4 * e + 1]) * f,
+                                            __uint_as_float(xo[4 * e + 2]) * f, __uint_as_float(xo[4 * e + 3]) * f);
+                        __syncwarp();
+#pragma unroll
+                        for (int it = 0; it < 8; ++it) {
+                            const int rw = it * 4 + (lane >> 3);  // row of the warp this lane writes
+                            float *d = reinterpret_cast<float *>(
+                                __shfl_sync(0xffffffffu, reinterpret_cast<unsigned long long>(dst), rw));
+                            const float4 val = *reinterpret_cast<const float4 *>(stage + rw * 36 + (lane & 7) * 4);
+                            if ((vmask >> rw) & 1u) *reinterpret_cast<float4 *>(d + ch * 32 + (lane & 7) * 4) = val;
                         }
+                        __syncwarp();
                     }
                     if (valid) {
                         const float m_nat = m_used * 0.6931471805599453f;
