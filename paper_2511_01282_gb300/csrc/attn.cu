@@ -286,6 +286,23 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
+// q [R, Hq, D] bf16 viewed as (D, Hq, R); boxes of 64 head-dim columns x G
+// heads x 128 / G nodes: one 128-row tile of (node, q-head-in-group) rows
+// in the order of the two-tile form, 128-byte swizzled (the K-major layout
+// the S MMA reads), zero fill past R.
+bool make_q_map(CUtensorMap *m, const void *base, int R, int Hq, int G, int D) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)Hq, (cuuint64_t)R};
+    cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)Hq * D * 2};
+    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)(kBM / G)};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 // [kv_rows, Hkv, D] bf16 viewed as a 3-D tensor (D, Hkv, kv_rows); boxes of
 // 64 head-dim columns x 1 head x 128 keys, 128-byte swizzled, zero fill.
 bool make_kv_map(CUtensorMap *m, const void *base, long long kv_rows, int Hkv, int D) {
@@ -389,6 +406,7 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     a.part_m = cv.take<float>(2 * (size_t)Gc * seg_rows);
     a.part_l = cv.take<float>(2 * (size_t)Gc * seg_rows);
     a.seg_rows = seg_rows;
+    a.q_tma = 0;
     a.jobs = cv.take<CombJob>((size_t)Gc);
     a.ranges = cv.take<int2>((size_t)Gc);
     a.B = B;
@@ -422,6 +440,19 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     cudaGetDevice(&dev);
     const int di = D == 128 ? 1 : 0;
     const bool pair = seg_rows == kPairRows;
+    // the two-tile form copies its Q tiles with TMA when a tile is whole
+    // nodes (G divides 128); otherwise its softmax threads write them
+    CUtensorMap tmq = tmk;  // never read unless a.q_tma
+    const int Gq = Hq / Hkv;
+    if (pair && R > 0 && kBM % Gq == 0) {
+        if (!make_q_map(&tmq, q, R, Hq, Gq, D)) {
+            set_error("rs_tree_verify_attn: cuTensorMapEncodeTiled (q) failed");
+            return RS_ERR_CUDA;
+        }
+        a.q_tma = 1;
+    }
+    if (const char *e = getenv("RS_DEBUG_ATTN_QCOPY"))  // test hook: force the thread-written Q path
+        if (!strcmp(e, "threads")) a.q_tma = 0;
     if (pair && dev >= 0 && dev < 64 && g_pair_regs_ok[dev][di] == 0) {
         // The two-tile kernel moves registers between its warpgroups with
         // setmaxnreg, sized for a launch of 168 registers per thread; with
@@ -466,9 +497,9 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     if (pair) {
         const size_t smem = attn_pair_smem_bytes(B);
         if (D == 128)
-            launch_full(attn_pair_kernel<128>, dim3(Gc), dim3(kPairThreads), smem, st, a, info, tmk, tmv);
+            launch_full(attn_pair_kernel<128>, dim3(Gc), dim3(kPairThreads), smem, st, a, info, tmk, tmv, tmq);
         else
-            launch_full(attn_pair_kernel<64>, dim3(Gc), dim3(kPairThreads), smem, st, a, info, tmk, tmv);
+            launch_full(attn_pair_kernel<64>, dim3(Gc), dim3(kPairThreads), smem, st, a, info, tmk, tmv, tmq);
     } else {
         const size_t smem = attn_smem_bytes(B);
         if (D == 128)

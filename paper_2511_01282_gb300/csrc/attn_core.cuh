@@ -102,6 +102,7 @@ struct AttnArgs {
     int2 *ranges;   // [gridDim.x]: each CTA's unit range [x, y)
     int kv_stream;  // the launch's K/V is large next to L2: stream tiles read once
     int seg_rows;   // rows per segment and per partial slot: 128, or 256 in the two-tile form
+    int q_tma;      // two-tile form: Q tiles are copied by TMA (128 % (Hq / Hkv) == 0)
     long long wait_limit;  // clock cycles a pipeline wait may take before the CTA gives up
     int B, Hq, Hkv, D;
     float scale;

@@ -28,6 +28,10 @@
 // written by the softmax threads) and S = Q K^T reads both operands from
 // shared memory; P stays in tensor memory for O += P V as in the one-tile
 // kernel.  K and V use a two-stage ring (a K/V tile now serves 256 rows).
+// When G = Hq / Hkv divides 128 a Q tile is whole nodes and the TMA warp
+// copies it (qfull / qfree barriers; the copy for the next piece starts as
+// soon as the tile's warps have finished their epilogue, which stages O rows
+// in the same buffer); otherwise the softmax threads write it (qready).
 //
 // Barrier phases: every role walks the same pieces in the same order and
 // counts, per S buffer, how many S it has held (use counts), so a wait's
@@ -55,7 +59,7 @@ constexpr int kP2SmemK = 0;
 constexpr int kP2SmemV = kP2SmemK + kPairNS * kTileBytes;
 constexpr int kP2SmemQ = kP2SmemV + kPairNS * kTileBytes;  // Q tile x at + x * kTileBytes
 constexpr int kP2SmemBar = kP2SmemQ + 2 * kTileBytes;
-constexpr int kP2NumBars = 6 * kPairNS + 3;
+constexpr int kP2NumBars = 6 * kPairNS + 7;
 constexpr int kP2SmemMisc = kP2SmemBar + kP2NumBars * 8;  // tmem base, abort flag
 constexpr int kP2SmemPref = kP2SmemMisc + 16;
 constexpr uint32_t kTm2S = 256;  // S/P buffer b at kTm2S + 128 b; O of tile x at 128 x
@@ -189,7 +193,7 @@ struct PairSplit {
 template <int D>
 __global__ void __launch_bounds__(kPairThreads, 1)
 attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_constant__ CUtensorMap tmk,
-                 const __grid_constant__ CUtensorMap tmv) {
+                 const __grid_constant__ CUtensorMap tmv, const __grid_constant__ CUtensorMap tmq) {
     pdl_launch_next();
     using namespace sm100;
     extern __shared__ unsigned char smem_raw[];
@@ -199,6 +203,7 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
     uint64_t *kfull = bars, *vfull = bars + kPairNS, *kempty = bars + 2 * kPairNS, *vempty = bars + 3 * kPairNS;
     uint64_t *sfull = bars + 4 * kPairNS, *pfull = sfull + 2;
     uint64_t *qready = pfull + 2, *ofree = qready + 1, *drain = ofree + 1;
+    uint64_t *qfull = drain + 1, *qfree = qfull + 2;  // Q tiles copied by TMA (a.q_tma)
     uint32_t *s_tmem = reinterpret_cast<uint32_t *>(smem + kP2SmemMisc);
     volatile int *s_abort = reinterpret_cast<volatile int *>(smem + kP2SmemMisc + 4);
     int *s_pref = reinterpret_cast<int *>(smem + kP2SmemPref);
@@ -218,6 +223,10 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
             mbar_init(&pfull[s], kBM);
         }
         mbar_init(qready, kSoftThreads);
+        for (int x = 0; x < 2; ++x) {
+            mbar_init(&qfull[x], 1);
+            mbar_init(&qfree[x], kBM);  // the tile's softmax warps, after their epilogue
+        }
         mbar_init(ofree, kSoftThreads);
         mbar_init(drain, 1);
         *s_abort = 0;
@@ -227,6 +236,7 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
     if (warp == kTmaWarp && lane == 0) {
         prefetch_tmap(&tmk);
         prefetch_tmap(&tmv);
+        if (a.q_tma) prefetch_tmap(&tmq);
     }
     pdl_wait_prev();  // the prologue above touches no global memory
     pair_prefix(info, a.B, a.Hkv, s_pref, s_spref, s_apref);  // contains __syncthreads
@@ -251,12 +261,15 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
         // ---------------------------------------------------------- TMA producer
         if (lane == 0) {
             uint32_t g = 0;
+            uint32_t quse[2] = {0, 0};  // Q tiles copied into buffers A and B so far
             bool ok = true;
             const uint64_t once = l2_evict_first_policy();
             for (long long u = u0; u < u1 && ok;) {
                 const Piece pc = piece_at(info, s_pref, a.B, u, u0, u1, c);
                 const long long kv0 = a.kv_off[pc.b];
-                const bool reread = !a.kv_stream || info[pc.b].mt > 1;  // kept in L2
+                const ReqInfo ri = info[pc.b];
+                const bool reread = !a.kv_stream || ri.mt > 1;  // kept in L2
+                const bool full = ri.rows - pc.mtile * kPairRows > kBM;
                 for (int jt = pc.j0; jt < pc.j1; ++jt, ++g) {
                     const int st = (int)(g & 1);
                     const uint32_t free_par = ((g >> 1) & 1) ^ 1;
@@ -281,6 +294,27 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
                         if (reread) tma_load_3d(sv + kb * 16384, &tmv, &vfull[st], kb * 64, pc.kvh, row);
                         else tma_load_3d_hint(sv + kb * 16384, &tmv, &vfull[st], kb * 64, pc.kvh, row, once);
                     }
+                    if (a.q_tma && jt == (pc.j1 - pc.j0 >= 2 ? pc.j0 + 1 : pc.j0)) {
+                        // the piece's Q tiles, once its first two K/V copies are
+                        // under way (they wait only for ring stages), each after
+                        // its buffer's previous piece has left it: rows (node,
+                        // head in group) of 128 / G nodes x G heads, the layout
+                        // the S MMA reads; rows past the request's end belong to
+                        // no output and are never stored
+                        const int node0 = a.node_off[pc.b] + (pc.mtile * kPairRows) / G;
+                        for (int x = 0; x < (full ? 2 : 1) && ok; ++x) {
+                            if (quse[x] > 0 &&
+                                !(ok = mbar_wait(&qfree[x], (quse[x] - 1) & 1, s_abort, a.wait_limit)))
+                                break;
+                            ++quse[x];
+                            mbar_expect_tx(&qfull[x], (uint32_t)kBM * D * 2);
+#pragma unroll
+                            for (int kb = 0; kb < kKB; ++kb)
+                                tma_load_3d(smem + kP2SmemQ + x * kTileBytes + kb * 16384, &tmq, &qfull[x], kb * 64,
+                                            pc.kvh * G, node0 + x * (kBM / G));
+                        }
+                        if (!ok) break;
+                    }
                 }
                 u = pc.end;
             }
@@ -290,6 +324,11 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
                     mbar_wait(&kfull[t & 1], (t >> 1) & 1, &no_abort, kWaitLimit);
                     mbar_wait(&vfull[t & 1], (t >> 1) & 1, &no_abort, kWaitLimit);
                 }
+                for (int x = 0; x < 2; ++x)
+                    if (quse[x] > 0) {
+                        volatile int no_abort = 0;
+                        mbar_wait(&qfull[x], (quse[x] - 1) & 1, &no_abort, kWaitLimit);
+                    }
             }
         }
         __syncwarp();
@@ -329,6 +368,7 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
             constexpr uint32_t kTileDesc = kTileBytes >> 4;
             uint32_t g = 0;             // KV tiles of the CTA so far
             uint32_t use0 = 0, use1 = 0;  // S held so far by S/P buffers 0 and 1
+            uint32_t quse0 = 0, quse1 = 0;  // Q tiles received in buffers A and B
             int piece = 0;
             bool ok = true;
             // S of tile t (stage t & 1) for row tile xq into buffer buf
@@ -358,7 +398,14 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
                 const Piece pc = piece_at(info, s_pref, a.B, u, u0, u1, c);
                 const int n = pc.j1 - pc.j0;
                 const bool full = info[pc.b].rows - pc.mtile * kPairRows > kBM;
-                if (!(ok = mbar_wait(qready, (uint32_t)(piece & 1), s_abort, a.wait_limit))) break;
+                if (a.q_tma) {  // the piece's Q tiles have landed
+                    if (!(ok = mbar_wait(&qfull[0], quse0 & 1, s_abort, a.wait_limit))) break;
+                    if (full && !(ok = mbar_wait(&qfull[1], quse1 & 1, s_abort, a.wait_limit))) break;
+                    ++quse0;
+                    quse1 += full ? 1 : 0;
+                } else if (!(ok = mbar_wait(qready, (uint32_t)(piece & 1), s_abort, a.wait_limit))) {
+                    break;
+                }
                 if (!(ok = mbar_wait(&kfull[g & 1], (g >> 1) & 1, s_abort, a.wait_limit))) break;
                 tc_fence_after();
                 issue_s(g, 0, 0);
@@ -444,7 +491,7 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
             const int S = a.ctx_len[pc.b];
             const int i = valid ? rr / G : 0;
             const int h = pc.kvh * G + (valid ? rr - i * G : 0);
-            if (active) {
+            if (active && !a.q_tma) {
                 // Q row -> shared memory, K-major with the 128-byte swizzle: the
                 // 16-byte chunk c of 64-column block kb of row r sits at
                 // kb * 16384 + r * 128 + ((c ^ (r & 7)) * 16)
@@ -457,7 +504,7 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
                     *reinterpret_cast<uint4 *>(qs + (e >> 3) * 16384 + r * 128 + (((e & 7) ^ (r & 7)) << 4)) = v[e];
                 fence_async_smem();
             }
-            warp_arrive(qready);
+            if (!a.q_tma) warp_arrive(qready);
             if (active) {
                 float m_used = -INFINITY, l = 0.f;
                 for (int tl = 0; tl < n; ++tl) {
@@ -617,6 +664,10 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
                     tc_fence_before();
                 }
                 if (!ok) break;
+                if (a.q_tma) {  // this tile's Q buffer (staging included) is free for the next copy
+                    fence_async_smem();
+                    warp_arrive(&qfree[x]);
+                }
             }
             if (full) {
                 use0 += n;

@@ -6,7 +6,8 @@ KV head, and the one-tile form otherwise.  RS_DEBUG_ATTN_FORM=one|pair
 forces either, so each is checked against the oracle on every (node, head)
 row of shapes that exercise its paths: full pairs, half pairs (a request of
 one tile, or the last pair of an odd tile count), segments split over
-several CTAs, head dims 64 and 128, GQA groups 1-16, masks crossing tiles,
+several CTAs, head dims 64 and 128, GQA groups 1-16 (Q tiles copied by
+TMA) and 5 (Q tiles written by the softmax threads), masks crossing tiles,
 rejected requests, many requests, and the bounded-wait time-out.
 """
 import numpy as np
@@ -45,13 +46,20 @@ SHAPES = [
     # no GQA (group 1): every request is one half pair
     dict(seed=25, B=4, Hq=8, Hkv=8, D=128, V=512, ctx=(100, 700), model_nodes=(10, 40), n_chains=(1, 2),
          chain_len=5),
+    # group 5 (does not divide 128): the softmax threads write the Q tiles
+    dict(seed=26, B=2, Hq=20, Hkv=4, D=128, V=512, ctx=(800, 1500), model_nodes=(90, 120), n_chains=(1, 3),
+         chain_len=8),
 ]
 
 
-@pytest.mark.parametrize("form", ["pair", "one"])
+# "pair" copies Q tiles with TMA where the group divides 128; "pair-threads"
+# forces the thread-written Q tiles (RS_DEBUG_ATTN_QCOPY=threads) everywhere
+@pytest.mark.parametrize("form", ["pair", "pair-threads", "one"])
 @pytest.mark.parametrize("kw", SHAPES, ids=[str(i) for i in range(len(SHAPES))])
 def test_forms_every_row(kw, form, monkeypatch):
-    monkeypatch.setenv("RS_DEBUG_ATTN_FORM", form)
+    monkeypatch.setenv("RS_DEBUG_ATTN_FORM", form.split("-")[0])
+    if form == "pair-threads":
+        monkeypatch.setenv("RS_DEBUG_ATTN_QCOPY", "threads")
     kw = dict(kw)
     seed = kw.pop("seed")
     w = synth.build(synth.small_spec(**kw), seed=seed)
