@@ -168,6 +168,15 @@ __device__ inline void unit_prefix(const ReqInfo *__restrict__ info, int B, int 
     __syncthreads();
 }
 
+// floor(a * b / d) for a, b >= 0 and d > 0, in 32-bit arithmetic whenever
+// the product fits (64-bit division is a long instruction sequence, and the
+// work split sits on every CTA's path to its first tile).
+__device__ __forceinline__ long long muldiv(long long a, long long b, long long d) {
+    const unsigned long long p = (unsigned long long)a * (unsigned long long)b;
+    if ((p >> 32) == 0 && d <= 0xffffffffll) return (long long)((uint32_t)p / (uint32_t)d);
+    return (long long)(p / (unsigned long long)d);
+}
+
 // last b with s_pref[b] <= u (so that request b owns unit u)
 __device__ __forceinline__ int find_req(const int *s_pref, int B, long long u) {
     int lo = 0, hi = B - 1;
@@ -203,8 +212,8 @@ struct Split {
         return pref[lo] + seg * nt + (off > 0 ? off : 0);
     }
     __device__ __forceinline__ long long range_lo(long long c) const {
-        if (beta == 0) return c * pref[B] / G;  // an even split of the units
-        return unit_at((int)(c * cost(B) / G));
+        if (beta == 0) return muldiv(c, pref[B], G);  // an even split of the units
+        return unit_at((int)muldiv(c, cost(B), G));
     }
     // The CTA holding the last unit of segment [s0, s1) of request b: that
     // unit's cost position x lies in CTA c's cost interval for

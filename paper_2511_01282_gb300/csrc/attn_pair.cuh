@@ -175,7 +175,7 @@ struct PairSplit {
         const int off = rem - beta;
         return pref[lo] + (long long)(kvh * r.mt + p) * r.nt + (off > 0 ? off / w : 0);
     }
-    __device__ __forceinline__ long long range_lo(long long c) const { return unit_at(c * cost(B) / G); }
+    __device__ __forceinline__ long long range_lo(long long c) const { return unit_at(muldiv(c, cost(B), G)); }
     // The CTA holding the last unit of segment [s0, s1) of request b: the
     // segment's cost interval ends at x_end, and CTA c's range holds the unit
     // at cost position x_end - 1 for c = (x_end G - 1) / C.
@@ -246,7 +246,7 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
     const long long Gc = gridDim.x, c = blockIdx.x;
     PairSplit split{s_pref, s_spref, s_apref, a.B, 0, (int)Gc, a.Hkv};
     {
-        int beta = (int)(W / (2 * Gc));
+        int beta = (int)muldiv(W, 1, 2 * Gc);
         if (beta > kSegCostMax) beta = kSegCostMax;
         split.beta = 2 * beta;  // in the weighted units (a half-pair unit weighs 2)
     }
