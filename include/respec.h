@@ -233,7 +233,10 @@ rs_status rs_match_scan(const int32_t *tokens, const int64_t *tok_off, int B,
  *            (j < ctx_len[b]) is row kv_off[b] + j and its tree node i is row
  *            kv_off[b] + ctx_len[b] + i.  k and v must be 16-byte aligned.
  *   kv_off   [B] int64;  ctx_len [B] int32 (>= 0);  node_off [B+1] int32;
- *            B <= 3840 requests per call; kv_rows < 2^31.
+ *            B <= 3840 requests per call; kv_rows < 2^31 and
+ *            (2 Hq + Hkv) (kv_rows / 128 + B) < 2.2e8 (the work split's
+ *            32-bit prefixes; RS_ERR_UNSUPPORTED otherwise, far beyond a KV
+ *            cache that fits in memory at common head counts).
  *   parents  [R] int32 local parent index per node; parents of node 0 is -1,
  *            0 <= parents[i] < i otherwise.
  *   D in {64, 128}; Hq a multiple of Hkv (grouped-query heads h share KV

@@ -328,8 +328,20 @@ int g_pair_regs_ok[64][2] = {};    // two-tile form: 1 usable, -1 not (register 
 // more (node, q-head-in-group) rows per request and KV head than one tile.
 // RS_DEBUG_ATTN_FORM=one|pair overrides the choice (a test hook: both forms
 // compute the same function).
-int attn_seg_rows(int B, int R, int Hq, int Hkv, int D) {
-    const bool pair_ok = B <= kPairMaxB;
+// The work split keeps its unit and cost prefixes in 32-bit integers.  A
+// request of N <= 256 nodes has at most (N G / 128 + 1) <= 2 G + 1 row tiles
+// per KV head and (S + N) / 128 + 1 KV tiles, so a call's units are below
+// (2 Hq + Hkv) (kv_rows / 128 + B); a unit costs at most 1 + kSegCostMax
+// (one-tile form) or kPairWF + kPairWH kSegCostMax (two-tile form) in the
+// split, and the costs must stay below 2^31.
+double attn_units_bound(int B, long long kv_rows, int Hq, int Hkv) {
+    return (2.0 * Hq + Hkv) * ((double)kv_rows / kBN + B);
+}
+constexpr double kSplitRange = 2.0e9;
+constexpr double kOneCost = 1 + kSegCostMax, kPairCost = kPairWF + kPairWH * kSegCostMax;
+
+int attn_seg_rows(int B, int R, int Hq, int Hkv, int D, long long kv_rows) {
+    const bool pair_ok = B <= kPairMaxB && attn_units_bound(B, kv_rows, Hq, Hkv) * kPairCost < kSplitRange;
     if (const char *e = getenv("RS_DEBUG_ATTN_FORM")) {
         if (!strcmp(e, "pair")) return pair_ok ? kPairRows : kBM;
         if (!strcmp(e, "one")) return kBM;
@@ -348,7 +360,9 @@ static int attn_grid() { return std::min(num_sms(), kAttnMaxGrid); }
 extern "C" size_t rs_tree_verify_attn_workspace_size(int B, int R, int Hq, int Hkv, int D) {
     if (B < 0 || R < 0 || Hq < 1 || Hkv < 1 || (D != 64 && D != 128)) return 0;
     const size_t Gc = (size_t)attn_grid();
-    const size_t rows = (size_t)attn_seg_rows(B, R, Hq, Hkv, D);
+    // sized for the two-tile form whenever the call could take it (the call
+    // itself may still fall back to the one-tile form on a huge KV cache)
+    const size_t rows = (size_t)attn_seg_rows(B, R, Hq, Hkv, D, 0);
     Carve cv(nullptr);
     cv.take<ReqInfo>((size_t)B);
     cv.take<uint32_t>((size_t)R * kAncWords);
@@ -386,13 +400,18 @@ extern "C" rs_status rs_tree_verify_attn(const uint16_t *q, const uint16_t *k, c
     RS_CHECK_ARG((((uintptr_t)out | (uintptr_t)workspace) & 15) == 0,
                  "rs_tree_verify_attn: out and workspace must be 16-byte aligned");
     if (B == 0) return RS_OK;
+    if (attn_units_bound(B, kv_rows, Hq, Hkv) * kOneCost >= kSplitRange) {
+        set_error("rs_tree_verify_attn: call too large for one launch's 32-bit work split "
+                  "((2 Hq + Hkv) (kv_rows / 128 + B) must stay below 2.2e8)");
+        return RS_ERR_UNSUPPORTED;
+    }
     const size_t need = rs_tree_verify_attn_workspace_size(B, R, Hq, Hkv, D);
     if (workspace_bytes < need || !workspace) {
         set_error("rs_tree_verify_attn: workspace %zu bytes < %zu required", workspace_bytes, need);
         return RS_ERR_CAPACITY;
     }
     const int Gc = attn_grid();
-    const int seg_rows = attn_seg_rows(B, R, Hq, Hkv, D);
+    const int seg_rows = attn_seg_rows(B, R, Hq, Hkv, D, kv_rows);
     Carve cv(workspace);
     ReqInfo *info = cv.take<ReqInfo>((size_t)B);
     uint32_t *anc = cv.take<uint32_t>((size_t)R * kAncWords);

@@ -47,10 +47,14 @@ namespace rs {
 
 constexpr int kPairRows = 2 * kBM;  // rows per segment
 constexpr int kPairNS = 2;          // K/V ring stages
-// cost weights of a KV tile in the work split: a full pair runs two row tiles
-// on it, a half pair one (the tile-A softmax of a half pair is not hidden
-// behind a second tile's MMAs, so it costs more than half a full pair)
-constexpr int kPairWF = 3, kPairWH = 2;
+// Cost weights of a K/V tile in the work split: a full pair runs two row
+// tiles on it, a half pair one.  When K/V tiles come from L2 (re-read by
+// several pairs) the tile costs its compute: clock stamps measured 3.43 k and
+// 1.92 k cycles (ratio 1.79, weights 9 : 5); when they stream from HBM once
+// (kv_stream) a tile costs mostly its bytes, the same for both, and 3 : 2
+// measured best (batched: 107.4 against 111.1 us with 9 : 5).
+constexpr int kPairWF = 9, kPairWH = 5;              // the larger pair, for bounds
+constexpr int kPairWFStream = 3, kPairWHStream = 2;
 constexpr int kPairMaxB = 2048;  // requests per call in this form (three prefixes in shared memory)
 constexpr int kPairThreads = 384;
 constexpr uint32_t kPairRegsSoft = 216, kPairRegsProd = 72;
@@ -67,10 +71,10 @@ constexpr uint32_t kTm2S = 256;  // S/P buffer b at kTm2S + 128 b; O of tile x a
 inline size_t attn_pair_smem_bytes(int B) { return 1024 + kP2SmemPref + 3 * (size_t)(B + 1) * sizeof(int); }
 
 // Exclusive prefixes over the requests of their units (s_pref), segments
-// (s_spref) and weighted units (s_apref: kPairWF per unit of a full pair,
-// kPairWH per unit of a half pair).
-__device__ inline void pair_prefix(const ReqInfo *__restrict__ info, int B, int Hkv, int *s_pref, int *s_spref,
-                                   int *s_apref) {
+// (s_spref) and weighted units (s_apref: wf per unit of a full pair, wh per
+// unit of a half pair).
+__device__ inline void pair_prefix(const ReqInfo *__restrict__ info, int B, int Hkv, int wf, int wh, int *s_pref,
+                                   int *s_spref, int *s_apref) {
     __shared__ int s_carry[3];
     __shared__ int s_w[3][32];
     if (threadIdx.x == 0) s_carry[0] = s_carry[1] = s_carry[2] = 0;
@@ -86,7 +90,7 @@ __device__ inline void pair_prefix(const ReqInfo *__restrict__ info, int B, int 
                 v[0] = ri.units;
                 v[1] = ri.units / ri.nt;
                 const bool last_half = ri.rows - (ri.mt - 1) * kPairRows <= kBM;
-                v[2] = kPairWF * ri.units - (last_half ? (kPairWF - kPairWH) * Hkv * ri.nt : 0);
+                v[2] = wf * ri.units - (last_half ? (wf - wh) * Hkv * ri.nt : 0);
             }
         }
         int x[3] = {v[0], v[1], v[2]};
@@ -134,11 +138,11 @@ __device__ inline void pair_prefix(const ReqInfo *__restrict__ info, int B, int 
 // The work split of the pair form: the one-tile form's cost split with
 // weighted units.  Request b occupies cost positions [cost(b), cost(b + 1)),
 // cost(b) = apref[b] + beta spref[b]; within it the KV heads follow each
-// other, and within a KV head its pairs, each costing nt w + beta (w =
-// kPairWF, or kPairWH for a half pair, which can only be the last).
+// other, and within a KV head its pairs, each costing nt w + beta (w = wf,
+// or wh for a half pair, which can only be the last).
 struct PairSplit {
     const int *pref, *spref, *apref;
-    int B, beta, G, Hkv;
+    int B, beta, G, Hkv, wf, wh;
     struct Req {
         int nt, mt;
         bool last_half;
@@ -150,9 +154,9 @@ struct PairSplit {
         const int units = pref[b + 1] - pref[b], segs = spref[b + 1] - spref[b];
         r.nt = units / segs;
         r.mt = segs / Hkv;
-        r.last_half = apref[b + 1] - apref[b] < kPairWF * units;
-        r.cF = r.nt * kPairWF + beta;
-        r.cL = r.nt * (r.last_half ? kPairWH : kPairWF) + beta;
+        r.last_half = apref[b + 1] - apref[b] < wf * units;
+        r.cF = r.nt * wf + beta;
+        r.cL = r.nt * (r.last_half ? wh : wf) + beta;
         r.ck = (r.mt - 1) * r.cF + r.cL;
         return r;
     }
@@ -171,7 +175,7 @@ struct PairSplit {
         int p = rem / r.cF;
         if (p > r.mt - 1) p = r.mt - 1;
         rem -= p * r.cF;
-        const int w = (p == r.mt - 1 && r.last_half) ? kPairWH : kPairWF;
+        const int w = (p == r.mt - 1 && r.last_half) ? wh : wf;
         const int off = rem - beta;
         return pref[lo] + (long long)(kvh * r.mt + p) * r.nt + (off > 0 ? off / w : 0);
     }
@@ -183,7 +187,7 @@ struct PairSplit {
         const Req r = req(b);
         const int sg = (int)((s0 - pref[b]) / r.nt);
         const int kvh = sg / r.mt, p = sg - kvh * r.mt;
-        const int w = (p == r.mt - 1 && r.last_half) ? kPairWH : kPairWF;
+        const int w = (p == r.mt - 1 && r.last_half) ? wh : wf;
         const long long x_end = (long long)cost(b) + (long long)kvh * r.ck + (long long)p * r.cF + beta + r.nt * w;
         return (x_end * G - 1) / cost(B);
     }
@@ -239,16 +243,17 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
         if (a.q_tma) prefetch_tmap(&tmq);
     }
     pdl_wait_prev();  // the prologue above touches no global memory
-    pair_prefix(info, a.B, a.Hkv, s_pref, s_spref, s_apref);  // contains __syncthreads
+    const int wf = a.kv_stream ? kPairWFStream : kPairWF, wh = a.kv_stream ? kPairWHStream : kPairWH;
+    pair_prefix(info, a.B, a.Hkv, wf, wh, s_pref, s_spref, s_apref);  // contains __syncthreads
     tc_fence_after();
     const uint32_t tmem = *s_tmem;
     const long long W = s_pref[a.B];
     const long long Gc = gridDim.x, c = blockIdx.x;
-    PairSplit split{s_pref, s_spref, s_apref, a.B, 0, (int)Gc, a.Hkv};
+    PairSplit split{s_pref, s_spref, s_apref, a.B, 0, (int)Gc, a.Hkv, wf, wh};
     {
         int beta = (int)muldiv(W, 1, 2 * Gc);
         if (beta > kSegCostMax) beta = kSegCostMax;
-        split.beta = 2 * beta;  // in the weighted units (a half-pair unit weighs 2)
+        split.beta = wh * beta;  // in the weighted units (a half-pair K/V tile weighs wh)
     }
     const long long u0 = split.range_lo(c), u1 = split.range_lo(c + 1);
     const int G = a.Hq / a.Hkv;

@@ -111,6 +111,10 @@ def test_bad_arguments_fail_before_launch(rs):
     # more requests than a call takes
     st = L.rs_tree_verify_attn(f, f, f, 10, f, f, f, f, 3841, 1, 4, 4, 128, 0.1, f, f, f, f, 1 << 30, None)
     assert st == rs.RS_ERR_INVALID_ARG and "3840" in rs.rs_last_error()
+    # a KV cache whose tile count could overflow the 32-bit work split is refused
+    st = L.rs_tree_verify_attn(f, f, f, (1 << 31) - 256, f, f, f, f, 1, 1, 64, 64, 128, 0.1, f, f, f, f, 1 << 30,
+                               None)
+    assert st == rs.RS_ERR_UNSUPPORTED and "32-bit work split" in rs.rs_last_error()
     # misaligned output rows or workspace
     st = L.rs_tree_verify_attn(f, f, f, 10, f, f, f, f, 1, 1, 4, 4, 128, 0.1, C.c_void_p(0x10004), f, f, f,
                                1 << 30, None)
