@@ -72,6 +72,13 @@ constexpr int kSegCostMax = 8;
 constexpr int kSegCostOff = 128;
 // unit and segment prefixes over the requests: 2 (B + 1) ints after kSmemPref
 inline size_t attn_smem_bytes(int B) { return 1024 + kSmemPref + 2 * (size_t)(B + 1) * sizeof(int); }
+// Epilogue staging (calls of at most kStageMaxB requests, where it fits):
+// per softmax warp 32 rows x 16 columns of O at a row stride of 20 floats,
+// after the prefixes (256-byte aligned).
+constexpr int kStageMaxB = 1024;
+constexpr int kStageFloats = 32 * 20;  // per warp
+__host__ __device__ inline size_t attn_stage_offset(int B) { return (kSmemPref + 2 * (size_t)(B + 1) * sizeof(int) + 255) & ~size_t(255); }
+inline size_t attn_smem_bytes_staged(int B) { return 1024 + attn_stage_offset(B) + 8 * kStageFloats * sizeof(float); }
 
 struct ReqInfo {
     int units;  // Hkv * mt * nt, 0 for a rejected request
@@ -102,6 +109,7 @@ struct AttnArgs {
     int2 *ranges;   // [gridDim.x]: each CTA's unit range [x, y)
     int kv_stream;  // the launch's K/V is large next to L2: stream tiles read once
     int seg_rows;   // rows per segment and per partial slot: 128, or 256 in the two-tile form
+    int stage;      // one-tile form: O rows leave through shared memory (attn_smem_bytes_staged)
     int q_tma;      // two-tile form: Q tiles are copied by TMA (128 % (Hq / Hkv) == 0)
     long long wait_limit;  // clock cycles a pipeline wait may take before the CTA gives up
     int B, Hq, Hkv, D;
@@ -650,10 +658,39 @@ attn_tc_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_consta
             tmem_wait_ld();
 #pragma unroll
             for (int ch = 0; ch < kHalfO / 32; ++ch) tmem_regs_ready(xo[ch]);
+            if (a.stage) {
+                // rows leave through shared memory so that a store instruction
+                // writes 8 rows x 64 contiguous bytes instead of 32 rows x 16:
+                // the warp stages 32 rows x 16 columns (row stride 20 floats,
+                // conflict-free writes), then each lane stores 4 columns of a row
+                float *dst = (pc.final ? a.out + orow * D : a.part_o + prow * D) + hw * kHalfO;
+                const unsigned vmask = __ballot_sync(0xffffffffu, valid);
+                float *stage = reinterpret_cast<float *>(smem + attn_stage_offset(a.B)) + warp * kStageFloats;
+#pragma unroll
+                for (int c16 = 0; c16 < kHalfO / 16; ++c16) {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const uint32_t *x = &xo[c16 >> 1][(c16 & 1) * 16 + 4 * e];
+                        *reinterpret_cast<float4 *>(stage + lane * 20 + 4 * e) =
+                            make_float4(__uint_as_float(x[0]) * f, __uint_as_float(x[1]) * f,
+                                        __uint_as_float(x[2]) * f, __uint_as_float(x[3]) * f);
+                    }
+                    __syncwarp();
+#pragma unroll
+                    for (int it = 0; it < 4; ++it) {
+                        const int rw = it * 8 + (lane >> 2);  // row of the warp this lane writes
+                        float *d = reinterpret_cast<float *>(
+                            __shfl_sync(0xffffffffu, reinterpret_cast<unsigned long long>(dst), rw));
+                        const float4 v4 = *reinterpret_cast<const float4 *>(stage + rw * 20 + (lane & 3) * 4);
+                        if ((vmask >> rw) & 1u) *reinterpret_cast<float4 *>(d + c16 * 16 + (lane & 3) * 4) = v4;
+                    }
+                    __syncwarp();
+                }
+            }
 #pragma unroll
             for (int ch = 0; ch < kHalfO / 32; ++ch) {
                 const int col = hw * kHalfO + ch * 32;
-                if (valid) {
+                if (valid && !a.stage) {
                     float4 *dst = pc.final ? reinterpret_cast<float4 *>(a.out + orow * D + col)
                                            : reinterpret_cast<float4 *>(a.part_o + prow * D + col);
 #pragma unroll
