@@ -166,7 +166,7 @@ def algorithmic_bytes(w):
 
 def attn_source_sha():
     h = hashlib.sha256()
-    for f in ("attn.cu", "attn_core.cuh"):
+    for f in ("attn.cu", "attn_core.cuh", "attn_pair.cuh", "sm100.cuh"):
         with open(os.path.join(ROOT, "paper_2511_01282_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
