@@ -153,3 +153,35 @@ def test_pair_form_time_out_reports_status_and_recovers(monkeypatch):
     q, k, v, kv_off, ctx, node_off, parents = inp
     ref = oracle.tree_attn(q, k, v, kv_off, ctx, node_off, parents, Hq, Hkv, D, D ** -0.5)
     assert np.abs(out.reshape(-1, D) - ref["out"]).max() < 1e-2
+
+
+def test_pair_form_empty_prefix_and_single_nodes(monkeypatch):
+    # requests with no committed prefix (the first tile is all tree slots)
+    # and single-node trees, in groups of 8 (half pairs and a full pair)
+    monkeypatch.setenv("RS_DEBUG_ATTN_FORM", "pair")
+    rng = np.random.default_rng(8)
+    Hq, Hkv, D = 16, 2, 128
+    trees = [[-1] + [int(rng.integers(0, i)) for i in range(1, 40)], [-1], [-1, 0, 1, 2], [-1],
+             [-1] + [int(rng.integers(0, i)) for i in range(1, 20)]]
+    S = [0, 0, 300, 1, 0]
+    inp = _attn_inputs(rng, Hq, Hkv, D, S, trees)
+    out, lse, status = _run_attn(*inp, Hq, Hkv, D, D ** -0.5)
+    assert (status == 0).all()
+    q, k, v, kv_off, ctx, node_off, parents = inp
+    ref = oracle.tree_attn(q, k, v, kv_off, ctx, node_off, parents, Hq, Hkv, D, D ** -0.5)
+    assert np.abs(out.reshape(-1, D) - ref["out"]).max() < 1e-2
+    assert np.abs(lse.reshape(-1) - ref["lse"]).max() < 1e-3
+
+
+def test_one_tile_form_streaming_launch_every_row(monkeypatch):
+    # K/V larger than half the L2 makes the launch stream it (evict-first
+    # copies, epilogue rows staged through shared memory): a small tree over
+    # long prefixes, every (node, head) row against the oracle
+    monkeypatch.setenv("RS_DEBUG_ATTN_FORM", "one")
+    kw = dict(B=2, Hq=8, Hkv=8, D=128, V=512, ctx=(20000, 22000), model_nodes=(20, 30), n_chains=(1, 2),
+              chain_len=6)
+    w = synth.build(synth.small_spec(**kw), seed=27)
+    kv_bytes = 2 * w.k.shape[0] * 8 * 128 * 2
+    l2 = getattr(torch.cuda.get_device_properties(0), "L2_cache_size", 129 * 2 ** 20)
+    assert kv_bytes > 0.5 * l2
+    check_attn(w, make_step(w), rows=None)
