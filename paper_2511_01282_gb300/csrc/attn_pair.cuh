@@ -49,12 +49,18 @@ constexpr int kPairRows = 2 * kBM;  // rows per segment
 constexpr int kPairNS = 2;          // K/V ring stages
 // Cost weights of a K/V tile in the work split: a full pair runs two row
 // tiles on it, a half pair one.  When K/V tiles come from L2 (re-read by
-// several pairs) the tile costs its compute: clock stamps measured 3.43 k and
-// 1.92 k cycles (ratio 1.79, weights 9 : 5); when they stream from HBM once
-// (kv_stream) a tile costs mostly its bytes, the same for both, and 3 : 2
-// measured best (batched: 107.4 against 111.1 us with 9 : 5).
-constexpr int kPairWF = 9, kPairWH = 5;              // the larger pair, for bounds
+// several pairs) the tile costs mostly its compute: a fit of per-CTA
+// lifetimes (global timer) on GQA-16K with a cold L2 gave 1.49 and 0.90 us
+// per full and half pair tile (weights 5 : 3; warm-L2 clock stamps, 3.43 k
+// and 1.92 k cycles, suggested 9 : 5).  When they stream from HBM once
+// (kv_stream) a tile costs mostly its bytes, the same for both: the fit on
+// the batched workload gave 1.61 and 1.09 us (3 : 2).  A segment start is
+// charged beta = min(cap, W / 2G) half-pair tiles: the fits put a piece
+// boundary at ~9 half-pair tiles from L2 and ~4 when streaming (the
+// streaming K/V copies run on through the boundary).
+constexpr int kPairWF = 5, kPairWH = 3;              // the larger pair, for bounds
 constexpr int kPairWFStream = 3, kPairWHStream = 2;
+constexpr int kPairSegCostStream = 4;  // the cap of beta when streaming (kSegCostMax otherwise)
 constexpr int kPairMaxB = 2048;  // requests per call in this form (three prefixes in shared memory)
 constexpr int kPairThreads = 384;
 constexpr uint32_t kPairRegsSoft = 216, kPairRegsProd = 72;
@@ -252,7 +258,8 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
     PairSplit split{s_pref, s_spref, s_apref, a.B, 0, (int)Gc, a.Hkv, wf, wh};
     {
         int beta = (int)muldiv(W, 1, 2 * Gc);
-        if (beta > kSegCostMax) beta = kSegCostMax;
+        const int cap = a.kv_stream ? kPairSegCostStream : kSegCostMax;
+        if (beta > cap) beta = cap;
         split.beta = wh * beta;  // in the weighted units (a half-pair K/V tile weighs wh)
     }
     const long long u0 = split.range_lo(c), u1 = split.range_lo(c + 1);
@@ -275,6 +282,11 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
                 const ReqInfo ri = info[pc.b];
                 const bool reread = !a.kv_stream || ri.mt > 1;  // kept in L2
                 const bool full = ri.rows - pc.mtile * kPairRows > kBM;
+                // Where K/V stays in L2 the CTA's first Q tiles follow its first
+                // K tile: every CTA starts at once and S needs only K and Q.
+                // Otherwise, and for later pieces, they follow the second K/V
+                // tile (below).
+                const bool q_early = a.q_tma && u == u0 && !a.kv_stream;
                 for (int jt = pc.j0; jt < pc.j1; ++jt, ++g) {
                     const int st = (int)(g & 1);
                     const uint32_t free_par = ((g >> 1) & 1) ^ 1;
@@ -288,6 +300,17 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
                         if (reread) tma_load_3d(sk + kb * 16384, &tmk, &kfull[st], kb * 64, pc.kvh, row);
                         else tma_load_3d_hint(sk + kb * 16384, &tmk, &kfull[st], kb * 64, pc.kvh, row, once);
                     }
+                    if (q_early && jt == pc.j0) {  // the buffers are unused: no wait
+                        const int node0 = a.node_off[pc.b] + (pc.mtile * kPairRows) / G;
+                        for (int x = 0; x < (full ? 2 : 1); ++x) {
+                            ++quse[x];
+                            mbar_expect_tx(&qfull[x], (uint32_t)kBM * D * 2);
+#pragma unroll
+                            for (int kb = 0; kb < kKB; ++kb)
+                                tma_load_3d(smem + kP2SmemQ + x * kTileBytes + kb * 16384, &tmq, &qfull[x], kb * 64,
+                                            pc.kvh * G, node0 + x * (kBM / G));
+                        }
+                    }
                     if (!(ok = mbar_wait(&vempty[st], free_par, s_abort, a.wait_limit))) {
                         volatile int no_abort = 0;  // this tile's K copy is in flight: let it land
                         mbar_wait(&kfull[st], (g >> 1) & 1, &no_abort, kWaitLimit);
@@ -299,7 +322,7 @@ attn_pair_kernel(AttnArgs a, const ReqInfo *__restrict__ info, const __grid_cons
                         if (reread) tma_load_3d(sv + kb * 16384, &tmv, &vfull[st], kb * 64, pc.kvh, row);
                         else tma_load_3d_hint(sv + kb * 16384, &tmv, &vfull[st], kb * 64, pc.kvh, row, once);
                     }
-                    if (a.q_tma && jt == (pc.j1 - pc.j0 >= 2 ? pc.j0 + 1 : pc.j0)) {
+                    if (a.q_tma && !q_early && jt == (pc.j1 - pc.j0 >= 2 ? pc.j0 + 1 : pc.j0)) {
                         // the piece's Q tiles, once its first two K/V copies are
                         // under way (they wait only for ring stages), each after
                         // its buffer's previous piece has left it: rows (node,
