@@ -17,6 +17,7 @@ Rank 0 prints one JSON line.
 """
 import argparse
 import hashlib
+import re
 import json
 import os
 import statistics
@@ -165,10 +166,16 @@ def algorithmic_bytes(w):
 
 
 def attn_source_sha():
+    """Hash of the attention kernels' sources with comments and blank space
+    taken out, so that a comment edit keeps the committed traffic records
+    while any change to the code retires them."""
     h = hashlib.sha256()
     for f in ("attn.cu", "attn_core.cuh", "attn_pair.cuh", "sm100.cuh"):
-        with open(os.path.join(ROOT, "paper_2511_01282_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2511_01282_gb300", "csrc", f)) as fh:
+            src = fh.read()
+        src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)   # block comments
+        src = re.sub(r"//[^\n]*", " ", src)                # line comments
+        h.update(" ".join(src.split()).encode())
     return h.hexdigest()[:16]
 
 

@@ -29,9 +29,11 @@
 // shared memory; P stays in tensor memory for O += P V as in the one-tile
 // kernel.  K and V use a two-stage ring (a K/V tile now serves 256 rows).
 // When G = Hq / Hkv divides 128 a Q tile is whole nodes and the TMA warp
-// copies it (qfull / qfree barriers; the copy for the next piece starts as
-// soon as the tile's warps have finished their epilogue, which stages O rows
-// in the same buffer); otherwise the softmax threads write it (qready).
+// copies it (qfull / qfree barriers): a CTA's first Q tiles right after its
+// first K tile when K/V stays in L2 (the buffers are still unused), all
+// others after the piece's second K/V tile, each once the tile's warps have
+// finished their epilogue, which stages O rows in the same buffer;
+// otherwise the softmax threads write it (qready).
 //
 // Barrier phases: every role walks the same pieces in the same order and
 // counts, per S buffer, how many S it has held (use counts), so a wait's
