@@ -324,7 +324,7 @@ int g_pair_regs_ok[64][2] = {};    // two-tile form: 1 usable, -1 not (register 
 
 // Rows per segment: 256 selects the two-row-tile form (attn_pair.cuh), which
 // pays off when requests have more than one 128-row tile per KV head.  The
-// host cannot see the trees, so it judges from the average over the call:
+// host cannot see the trees, so it decides from the average over the call:
 // more (node, q-head-in-group) rows per request and KV head than one tile.
 // RS_DEBUG_ATTN_FORM=one|pair overrides the choice (a test hook: both forms
 // compute the same function).

@@ -1,7 +1,8 @@
 """Shared parity checks: run the C-ABI calls on the GPU and compare each
 output with the oracle on the same seeded inputs.
 
-Tolerances (BASELINE north star, restated per output):
+Tolerances, per output (exact where the result is an integer or a decision,
+the arithmetic's rounding bound otherwise):
   * match positions, counts, spans, selections, argmax, top-beta ids,
     acceptance decisions, accepted paths, winners, bonus tokens, commit flags,
     status words and updated scores: bit-exact;
