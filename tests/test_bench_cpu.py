@@ -1,7 +1,8 @@
 """Host-side parts of bench.py on the CPU: the reference arm (the oracle timed
 on the host cores) prints one well-formed JSON line, and fanning the oracle's
 attention out over threads by row chunks returns exactly what one call over
-the same rows returns (each row is computed on its own)."""
+the same rows returns (each row is computed on its own); the DRAM-traffic
+records follow the attention code, not its comments."""
 import json
 import os
 import subprocess
@@ -46,3 +47,23 @@ def test_threaded_oracle_attention_equals_one_call():
     # the benchmark's fan-out runs the same rows (it only times them)
     bench.oracle_attn_rows(w, rows[:17], workers=4)
     assert bench.host_cores() >= 1
+
+
+def test_traffic_records_follow_the_code_not_the_comments(tmp_path, monkeypatch):
+    # the committed DRAM-traffic records are keyed by a hash of the attention
+    # sources with comments and blank space taken out: a comment edit keeps
+    # them, any change to the code retires them
+    sys.path.insert(0, ROOT)
+    import bench
+    csrc = tmp_path / "paper_2511_01282_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    for f in ("attn.cu", "attn_core.cuh", "attn_pair.cuh", "sm100.cuh"):
+        (csrc / f).write_text(open(os.path.join(ROOT, "paper_2511_01282_gb300", "csrc", f)).read())
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    h0 = bench.attn_source_sha()
+    core = csrc / "attn_core.cuh"
+    src = core.read_text()
+    core.write_text(src.replace("namespace rs {", "// a new comment line\nnamespace rs {  /* and a block */", 1))
+    assert bench.attn_source_sha() == h0
+    core.write_text(src.replace("constexpr int kNS = 3;", "constexpr int kNS = 4;", 1))
+    assert bench.attn_source_sha() != h0
