@@ -185,3 +185,19 @@ def test_one_tile_form_streaming_launch_every_row(monkeypatch):
     l2 = getattr(torch.cuda.get_device_properties(0), "L2_cache_size", 129 * 2 ** 20)
     assert kv_bytes > 0.5 * l2
     check_attn(w, make_step(w), rows=None)
+
+
+def test_pair_form_streaming_launch_every_row(monkeypatch):
+    # K/V larger than half the L2 makes a pair-form launch stream it (evict-
+    # first copies, the streaming split weights, every CTA's first Q copied
+    # after its second K/V tile): GQA 4 over a few hundred tree nodes and long
+    # prefixes, every (node, head) row against the oracle
+    monkeypatch.setenv("RS_DEBUG_ATTN_FORM", "pair")
+    kw = dict(B=2, Hq=32, Hkv=8, D=128, V=512, ctx=(20000, 21000), model_nodes=(90, 110), n_chains=(1, 2),
+              chain_len=6)
+    w = synth.build(synth.small_spec(**kw), seed=28)
+    kv_bytes = 2 * w.k.shape[0] * 8 * 128 * 2
+    l2 = getattr(torch.cuda.get_device_properties(0), "L2_cache_size", 129 * 2 ** 20)
+    assert kv_bytes > 0.5 * l2
+    assert int(np.diff(w.node_off).max()) * 4 > 128  # more than one row tile per KV head
+    check_attn(w, make_step(w), rows=None)
