@@ -8,7 +8,8 @@ row of shapes that exercise its paths: full pairs, half pairs (a request of
 one tile, or the last pair of an odd tile count), segments split over
 several CTAs, head dims 64 and 128, GQA groups 1-16 (Q tiles copied by
 TMA) and 5 (Q tiles written by the softmax threads), masks crossing tiles,
-rejected requests, many requests, and the bounded-wait time-out.
+rejected requests, many requests, launches that stream K/V from HBM, and
+the bounded-wait time-out.
 """
 import numpy as np
 import pytest
