@@ -202,3 +202,27 @@ def test_pair_form_streaming_launch_every_row(monkeypatch):
     assert kv_bytes > 0.5 * l2
     assert int(np.diff(w.node_off).max()) * 4 > 128  # more than one row tile per KV head
     check_attn(w, make_step(w), rows=None)
+
+
+@pytest.mark.parametrize("form", ["pair", "one"])
+def test_row_counts_at_tile_edges(form, monkeypatch):
+    # (node, head-in-group) rows per KV head of exactly one tile, one tile and
+    # one node, exactly two tiles and two tiles and one node (G = 8: 16, 17,
+    # 32 and 33 nodes): half pairs, full pairs with a short second tile and
+    # pairs followed by a half pair, with prefixes that end on, just before
+    # and just after a 128-key boundary
+    monkeypatch.setenv("RS_DEBUG_ATTN_FORM", form)
+    rng = np.random.default_rng(9)
+    Hq, Hkv, D = 16, 2, 128
+    trees = []
+    for n in (16, 17, 32, 33):
+        trees.append([-1] + [int(rng.integers(max(0, i - 3), i)) for i in range(1, n)])
+    S = [256, 255, 257, 640]
+    inp = _attn_inputs(rng, Hq, Hkv, D, S, trees)
+    out, lse, status = _run_attn(*inp, Hq, Hkv, D, D ** -0.5)
+    assert (status == 0).all()
+    q, k, v, kv_off, ctx, node_off, parents = inp
+    ref = oracle.tree_attn(q, k, v, kv_off, ctx, node_off, parents, Hq, Hkv, D, D ** -0.5)
+    assert np.abs(out.reshape(-1, D) - ref["out"]).max() < 1e-2
+    assert np.linalg.norm(out.reshape(-1, D) - ref["out"]) / np.linalg.norm(ref["out"]) < 1e-2
+    assert np.abs(lse.reshape(-1) - ref["lse"]).max() < 1e-3
