@@ -154,3 +154,20 @@ def test_oracle_and_library_share_no_source():
     for fn in os.listdir(ora):
         if fn.endswith((".c", ".h")):
             assert "respec.h" not in open(os.path.join(ora, fn)).read()
+
+
+def test_attention_form_choice_sizes_the_workspace(rs, monkeypatch):
+    # the host picks the two-row-tile form (256-row partial slots) when the
+    # requests average more than one 128-row tile of (node, head-in-group)
+    # rows per KV head, and the workspace follows the choice: GQA 4 over 145
+    # nodes (580 rows per KV head) takes it, 40 KV heads over 65 nodes per
+    # request (65 rows) do not; RS_DEBUG_ATTN_FORM forces either
+    ws = rs.rs_tree_verify_attn_workspace_size
+    monkeypatch.delenv("RS_DEBUG_ATTN_FORM", raising=False)
+    g_def, o_def = ws(1, 145, 32, 8, 128), ws(4, 260, 40, 40, 128)
+    monkeypatch.setenv("RS_DEBUG_ATTN_FORM", "one")
+    g_one, o_one = ws(1, 145, 32, 8, 128), ws(4, 260, 40, 40, 128)
+    monkeypatch.setenv("RS_DEBUG_ATTN_FORM", "pair")
+    g_pair, o_pair = ws(1, 145, 32, 8, 128), ws(4, 260, 40, 40, 128)
+    assert g_def == g_pair > g_one
+    assert o_def == o_one < o_pair
